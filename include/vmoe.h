@@ -1,0 +1,191 @@
+/*
+ * vmoe.h -- C ABI of libvmoe: one adaptation step of T concurrent V-MoE expert
+ * layers on one NVIDIA GB300 (sm_103a).
+ *
+ * The method is AdaSprite's multi-task V-MoE co-adaptation (arxiv 2608.16188):
+ * the experts of T V-MoEs form one pool (Section 2.2, "MoE merging"); each
+ * task keeps its own router and experts and its tokens are routed to their
+ * most relevant experts (Section 2.1) under per-expert capacity limits
+ * (Challenge #1 in Section 1, Section 2.3.1); the experts of all tasks run
+ * concurrently (Section 3.2, expert parallelism) and only the visual
+ * experts are adapted (Section 3.1, specification-based tuning).  Here every
+ * stage is one grouped launch over all T*E (task, expert) groups.
+ *
+ * One step is:
+ *   vmoe_route     logits = x W_r + bias; softmax; top-k; capacity scan
+ *   vmoe_dispatch  Xe  = gather(x)               (padding rows zero)
+ *   vmoe_expert_fwd H = Xe W1, A = GELU(H), Ye = A W2
+ *   vmoe_combine   y   = sum_j gate_j * Ye[e_j, s_j]
+ *   vmoe_dispatch  dYe = gate * gather(dY)
+ *   vmoe_expert_bwd dH = (dYe W2^T) * GELU'(H), dXe = dH W1^T,
+ *                  dW1 = Xe^T dH, dW2 = A^T dYe
+ *   vmoe_combine   dX  = sum_j dXe[e_j, s_j]
+ *
+ * Conventions for every entry point:
+ *  - Ownership: every array argument is caller-owned DEVICE memory (except
+ *    the vmoe_problem struct, read on the host), row-major and contiguous in
+ *    the layout stated, with a base address aligned to 16 bytes.  The library
+ *    allocates no device memory and keeps no state between calls other than
+ *    the device status word (vmoe_device_status) and the optional trace.
+ *  - Execution: calls enqueue kernels on `cuda_stream` (a cudaStream_t; NULL
+ *    is the legacy default stream) and return without synchronising.
+ *  - Errors: arguments are checked on the host before any launch; an invalid
+ *    argument returns VMOE_ERR_INVALID and an unsupported shape
+ *    VMOE_ERR_UNSUPPORTED, in both cases with nothing launched.  A failed
+ *    launch returns VMOE_ERR_CUDA.  Device data (indices, loads) is trusted:
+ *    indices out of range are undefined behaviour.
+ *  - Determinism: results are bitwise reproducible run to run (no atomics in
+ *    any reduction, fixed summation orders).
+ *  - Dtypes: x, dY, weights and all activations use p->dtype (fp32 or bf16);
+ *    W_r, bias, logits and gates are always fp32.  bf16 contractions
+ *    accumulate in fp32 on the tcgen05 tensor cores; fp32 runs on CUDA cores.
+ *
+ * Shapes (t < T tasks, n < N tokens per task, e < E experts per task,
+ * j < k choices, s < C capacity slots, g = t*E + e):
+ *   x, y, dY, dX [T,N,d]   W_r [T,d,E]   bias [T,E]   logits [T,N,E]
+ *   expert_idx, gate, slot [T,N,k]   load [T,E]
+ *   Xe, Ye, dYe, dXe [T,E,C,d]   H, A [T,E,C,f]
+ *   W1, dW1 [T,E,d,f]   W2, dW2 [T,E,f,d]
+ */
+#ifndef VMOE_H
+#define VMOE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define VMOE_VERSION 1
+
+typedef enum {
+    VMOE_OK = 0,
+    VMOE_ERR_INVALID = -1,        /* bad argument; nothing launched */
+    VMOE_ERR_UNSUPPORTED = -2,    /* valid but unsupported shape; nothing launched */
+    VMOE_ERR_CUDA = -3,           /* a CUDA runtime call or launch failed */
+    VMOE_ERR_DEVICE_TIMEOUT = -4  /* a kernel gave up a bounded wait (vmoe_device_status) */
+} vmoe_status;
+
+typedef enum { VMOE_F32 = 0, VMOE_BF16 = 1 } vmoe_dtype;
+
+enum {
+    VMOE_LOGITS_IN = 1u << 0, /* vmoe_route reads `logits` instead of computing them */
+    VMOE_NO_RENORM = 1u << 1, /* gate = softmax probability (V-MoE); default renormalises over top-k */
+    VMOE_GELU_TANH = 1u << 2  /* tanh-approximate GELU; default is the exact erf form */
+};
+
+/* The problem statement: T tasks, each with N tokens of width d_model, its own
+ * router and E experts of hidden width d_ff; top-k routing with capacity
+ * C = ceil(capacity_factor * k * N / E) clamped to [1, N], or `capacity` when
+ * it is > 0.  Limits: T, N, E >= 1; 1 <= k <= min(E, 8); E <= 256;
+ * T*E <= 1024; d_model % 8 == 0.  The bf16 expert path also needs d_model and
+ * d_ff to be multiples of 128 (VMOE_ERR_UNSUPPORTED otherwise). */
+typedef struct {
+    int32_t T, N, d_model, d_ff, E, k;
+    double capacity_factor;
+    int32_t capacity;
+    vmoe_dtype dtype;
+    uint32_t flags;
+} vmoe_problem;
+
+/* Library version (VMOE_VERSION). */
+int vmoe_version(void);
+
+/* Human-readable name of a vmoe_status value (static storage). */
+const char *vmoe_status_string(int status);
+
+/* The capacity C the library uses for `p` (capacity rule above), or a negative
+ * vmoe_status if `p` is invalid.  Host only; no device work. */
+int vmoe_problem_capacity(const vmoe_problem *p);
+
+/* Routing: top-k softmax gating with per-expert capacity (Section 2.1 routing
+ * to the most relevant experts; capacity limits of Challenge #1; sequential
+ * assignment of Section 3.3.1).
+ *   x          [T,N,d] p->dtype           input tokens (unused with VMOE_LOGITS_IN; may be NULL then)
+ *   w_router   [T,d,E] fp32               per-task router (unused with VMOE_LOGITS_IN)
+ *   logit_bias [T,E]   fp32, nullable     per-task additive logit bias
+ *   logits     [T,N,E] fp32               output, or input with VMOE_LOGITS_IN
+ *   expert_idx [T,N,k] int32 out          the k largest logits, descending, ties to the lower index
+ *   gate       [T,N,k] fp32 out           softmax probability of each choice, divided by the
+ *                                         top-k probability mass unless VMOE_NO_RENORM
+ *   slot       [T,N,k] int32 out          position in the expert's buffer, -1 if dropped: in
+ *                                         choice-major order (all first choices in token order,
+ *                                         then all second choices, ...) the s-th assignment to an
+ *                                         expert gets slot s while s < C
+ *   load       [T,E]   int32 out          kept assignments per expert = min(count, C)
+ * Logits are accumulated in fp32.  A NaN logit is treated as -inf when the
+ * experts are chosen (indices stay in range); its gates are unspecified. */
+int vmoe_route(const vmoe_problem *p, const void *x, const float *w_router,
+               const float *logit_bias, float *logits, int32_t *expert_idx, float *gate,
+               int32_t *slot, int32_t *load, void *cuda_stream);
+
+/* Dispatch (permute into expert-contiguous buffers for the grouped expert
+ * launch of Section 3.2): dst[t,e,s,:] = w * src[t,n,:] for the kept choice
+ * (n, j) with expert_idx = e and slot = s, w = weight[t,n,j] or 1 if weight
+ * is NULL; rows s >= load[t,e] of dst are written as zero.
+ *   src [T,N,d] p->dtype, weight [T,N,k] fp32 nullable, expert_idx/slot [T,N,k],
+ *   load [T,E], dst [T,E,C,d] p->dtype (every element written).
+ * The weighted product is formed in fp32 and rounded to p->dtype. */
+int vmoe_dispatch(const vmoe_problem *p, const void *src, const float *weight,
+                  const int32_t *expert_idx, const int32_t *slot, const int32_t *load,
+                  void *dst, void *cuda_stream);
+
+/* Expert FFN forward over all T*E groups in one grouped launch per layer
+ * (Section 2.1: the ViT MLP block becomes experts; no bias terms):
+ *   H = Xe W1, A = GELU(H), Ye = A W2, per group g for its rows s < load[g].
+ *   xe [T,E,C,d], w1 [T,E,d,f], w2 [T,E,f,d], load [T,E] int32
+ *   h, a [T,E,C,f] out, ye [T,E,C,d] out -- rows s >= load[g] are not written.
+ * bf16: fp32 accumulation; A is GELU of the fp32 accumulator, H and A are
+ * stored rounded to bf16. */
+int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const void *w2,
+                    const int32_t *load, void *h, void *a, void *ye, void *cuda_stream);
+
+/* Device bytes of scratch vmoe_expert_bwd needs for `p` (the dH buffer,
+ * T*E*C*d_ff elements of p->dtype), or 0 if `p` is invalid.  Host only. */
+size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p);
+
+/* Expert FFN backward (adaptation of the expert weights, Section 3.1), the
+ * gradient of <dY, y> through the expert path with routing and gates fixed:
+ *   dH = (dYe W2^T) * GELU'(H), dXe = dH W1^T, dW1 = Xe^T dH, dW2 = A^T dYe,
+ * the weight gradients summing over each group's rows s < load[g].
+ *   xe [T,E,C,d], h, a [T,E,C,f] (from vmoe_expert_fwd), w1, w2, dye [T,E,C,d]
+ *   (= vmoe_dispatch(dY, gate)), load [T,E]
+ *   dxe [T,E,C,d] out (rows >= load not written), dw1 [T,E,d,f] out, dw2 [T,E,f,d] out
+ *   (every element written; zero for a group with load 0)
+ *   workspace: caller-owned device scratch of at least
+ *   vmoe_expert_bwd_workspace_size(p) bytes, 16-byte aligned; its contents are
+ *   clobbered.  Too small or NULL returns VMOE_ERR_INVALID. */
+int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,
+                    const void *w1, const void *w2, const void *dye, const int32_t *load,
+                    void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,
+                    void *cuda_stream);
+
+/* Combine back to token order: dst[t,n,:] = sum over kept choices j (slot >= 0)
+ * of w * src[t, expert_idx_j, slot_j, :], w = weight[t,n,j] or 1 if NULL,
+ * summed in fp32 in the order j = 0..k-1 and rounded once; a token with every
+ * choice dropped gets zero.
+ *   src [T,E,C,d], weight [T,N,k] fp32 nullable, expert_idx/slot [T,N,k],
+ *   dst [T,N,d] out.  The forward uses weight = gate, the backward (dX) NULL. */
+int vmoe_combine(const vmoe_problem *p, const void *src, const float *weight,
+                 const int32_t *expert_idx, const int32_t *slot, void *dst, void *cuda_stream);
+
+/* Device status word of the current device: 0 when clean, otherwise a
+ * vmoe_status (VMOE_ERR_DEVICE_TIMEOUT after a kernel gave up a bounded
+ * wait).  Synchronises the current device.  `reset` != 0 clears the word. */
+int vmoe_device_status(int reset);
+
+/* Kernel trace (host-side tracing aid).  While enabled on the calling host
+ * thread, every kernel the library launches is bracketed by two CUDA events
+ * recorded on its stream; at most `max_records` launches are kept.
+ * vmoe_trace_disable stops recording and returns the number of records;
+ * vmoe_trace_get synchronises on record i and returns its kernel name (static
+ * storage) and duration in milliseconds.  Returns VMOE_OK or a vmoe_status. */
+int vmoe_trace_enable(int max_records);
+int vmoe_trace_disable(void);
+int vmoe_trace_get(int i, const char **kernel_name, float *ms);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* VMOE_H */

@@ -1,0 +1,198 @@
+"""Python binding of libvmoe: one adaptation step of T concurrent V-MoE expert layers on GB300.
+
+Argument marshalling only.  Every step of the path runs in the CUDA kernels of
+``libvmoe.so`` (built in-tree by ``_build.build()``); there is no Python, PyTorch
+or CPU fallback, and importing a function whose library is missing raises.
+
+The functions carry the C names (``vmoe_route``, ``vmoe_dispatch``,
+``vmoe_expert_fwd``, ``vmoe_expert_bwd``, ``vmoe_combine``) and take torch tensors
+(device memory, any dtype matching the problem) or raw integer device pointers;
+``stream`` is a ``torch.cuda.Stream``, a raw ``cudaStream_t`` integer, or None for
+the current torch stream.  A non-zero status raises ``VmoeError``.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.environ.get("VMOE_LIBRARY", os.path.join(PKG, "libvmoe.so"))
+
+VMOE_OK = 0
+VMOE_ERR_INVALID = -1
+VMOE_ERR_UNSUPPORTED = -2
+VMOE_ERR_CUDA = -3
+VMOE_ERR_DEVICE_TIMEOUT = -4
+
+VMOE_F32 = 0
+VMOE_BF16 = 1
+
+VMOE_LOGITS_IN = 1 << 0
+VMOE_NO_RENORM = 1 << 1
+VMOE_GELU_TANH = 1 << 2
+
+# Every symbol include/vmoe.h declares.
+EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
+           "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
+           "vmoe_expert_bwd", "vmoe_combine", "vmoe_device_status", "vmoe_trace_enable",
+           "vmoe_trace_disable", "vmoe_trace_get")
+
+
+class VmoeError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        super().__init__("%s: %s" % (where, status_string(status)))
+
+
+class VmoeProblem(ctypes.Structure):
+    """Mirror of ``vmoe_problem`` in include/vmoe.h."""
+    _fields_ = [("T", ctypes.c_int32), ("N", ctypes.c_int32), ("d_model", ctypes.c_int32),
+                ("d_ff", ctypes.c_int32), ("E", ctypes.c_int32), ("k", ctypes.c_int32),
+                ("capacity_factor", ctypes.c_double), ("capacity", ctypes.c_int32),
+                ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+
+
+_lib = None
+_P = ctypes.c_void_p
+
+
+def library():
+    """The loaded libvmoe (ctypes.CDLL).  Raises if it has not been built."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                "libvmoe.so not found at %s: build it first with "
+                "`python -c 'import __graft_entry__ as g; g.build()'`" % LIB_PATH)
+        lib = ctypes.CDLL(LIB_PATH)
+        PP = ctypes.POINTER(VmoeProblem)
+        sig = {
+            "vmoe_version": (ctypes.c_int, []),
+            "vmoe_status_string": (ctypes.c_char_p, [ctypes.c_int]),
+            "vmoe_problem_capacity": (ctypes.c_int, [PP]),
+            "vmoe_route": (ctypes.c_int, [PP] + [_P] * 8 + [_P]),
+            "vmoe_dispatch": (ctypes.c_int, [PP] + [_P] * 6 + [_P]),
+            "vmoe_expert_fwd": (ctypes.c_int, [PP] + [_P] * 7 + [_P]),
+            "vmoe_expert_bwd_workspace_size": (ctypes.c_size_t, [PP]),
+            "vmoe_expert_bwd": (ctypes.c_int, [PP] + [_P] * 11 + [ctypes.c_size_t, _P]),
+            "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
+            "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
+            "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
+            "vmoe_trace_disable": (ctypes.c_int, []),
+            "vmoe_trace_get": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
+                                              ctypes.POINTER(ctypes.c_float)]),
+        }
+        for name, (res, args) in sig.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+    return _lib
+
+
+def status_string(status: int) -> str:
+    try:
+        return library().vmoe_status_string(int(status)).decode()
+    except Exception:  # library not loadable
+        return "status %d" % status
+
+
+def _ptr(t):
+    if t is None:
+        return None
+    if isinstance(t, int):
+        return t
+    return t.data_ptr()
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _check(st: int, where: str):
+    if st != VMOE_OK:
+        raise VmoeError(st, where)
+
+
+def problem(T, N, d_model, d_ff, E, k, capacity_factor, dtype="bf16", flags=0, capacity=0):
+    """Build a VmoeProblem; ``dtype`` is "bf16", "f32" or a VMOE_* code."""
+    if isinstance(dtype, str):
+        dtype = {"bf16": VMOE_BF16, "f32": VMOE_F32}[dtype]
+    return VmoeProblem(int(T), int(N), int(d_model), int(d_ff), int(E), int(k),
+                       float(capacity_factor), int(capacity), int(dtype), int(flags))
+
+
+def vmoe_version() -> int:
+    return library().vmoe_version()
+
+
+def vmoe_problem_capacity(p: VmoeProblem) -> int:
+    c = library().vmoe_problem_capacity(ctypes.byref(p))
+    if c < 0:
+        raise VmoeError(c, "vmoe_problem_capacity")
+    return c
+
+
+def vmoe_expert_bwd_workspace_size(p: VmoeProblem) -> int:
+    return int(library().vmoe_expert_bwd_workspace_size(ctypes.byref(p)))
+
+
+def vmoe_route(p, x, w_router, logit_bias, logits, expert_idx, gate, slot, load, stream=None):
+    _check(library().vmoe_route(ctypes.byref(p), _ptr(x), _ptr(w_router), _ptr(logit_bias),
+                                _ptr(logits), _ptr(expert_idx), _ptr(gate), _ptr(slot),
+                                _ptr(load), _stream(stream)), "vmoe_route")
+
+
+def vmoe_dispatch(p, src, weight, expert_idx, slot, load, dst, stream=None):
+    _check(library().vmoe_dispatch(ctypes.byref(p), _ptr(src), _ptr(weight), _ptr(expert_idx),
+                                   _ptr(slot), _ptr(load), _ptr(dst), _stream(stream)),
+           "vmoe_dispatch")
+
+
+def vmoe_expert_fwd(p, xe, w1, w2, load, h, a, ye, stream=None):
+    _check(library().vmoe_expert_fwd(ctypes.byref(p), _ptr(xe), _ptr(w1), _ptr(w2), _ptr(load),
+                                     _ptr(h), _ptr(a), _ptr(ye), _stream(stream)),
+           "vmoe_expert_fwd")
+
+
+def vmoe_expert_bwd(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2, workspace, workspace_bytes=None,
+                    stream=None):
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(library().vmoe_expert_bwd(ctypes.byref(p), _ptr(xe), _ptr(h), _ptr(a), _ptr(w1),
+                                     _ptr(w2), _ptr(dye), _ptr(load), _ptr(dxe), _ptr(dw1),
+                                     _ptr(dw2), _ptr(workspace), int(workspace_bytes),
+                                     _stream(stream)), "vmoe_expert_bwd")
+
+
+def vmoe_combine(p, src, weight, expert_idx, slot, dst, stream=None):
+    _check(library().vmoe_combine(ctypes.byref(p), _ptr(src), _ptr(weight), _ptr(expert_idx),
+                                  _ptr(slot), _ptr(dst), _stream(stream)), "vmoe_combine")
+
+
+def vmoe_device_status(reset: bool = False) -> int:
+    return library().vmoe_device_status(1 if reset else 0)
+
+
+def vmoe_trace_enable(max_records: int):
+    _check(library().vmoe_trace_enable(int(max_records)), "vmoe_trace_enable")
+
+
+def vmoe_trace_disable() -> int:
+    return library().vmoe_trace_disable()
+
+
+def vmoe_trace_get(i: int):
+    name = ctypes.c_char_p()
+    ms = ctypes.c_float()
+    _check(library().vmoe_trace_get(int(i), ctypes.byref(name), ctypes.byref(ms)),
+           "vmoe_trace_get")
+    return name.value.decode(), ms.value
+
+
+from .step import Buffers, StepRunner  # noqa: E402  (needs the names above)

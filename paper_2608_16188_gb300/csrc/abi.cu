@@ -1,0 +1,280 @@
+// abi.cu -- the extern "C" entry points of libvmoe: argument checks, capacity
+// rule, dtype selection, the device status word and the kernel trace.
+#include <math.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <vector>
+
+#include "common.cuh"
+
+namespace vmoe {
+
+// One status word per device that loads the library.  Kernels that give up a
+// bounded wait OR a vmoe_status into it; vmoe_device_status reads it.
+static __device__ int g_status_word = 0;
+
+int *device_status_word() {
+    static int *addr[64] = {nullptr};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+    if (!addr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
+        addr[dev] = static_cast<int *>(p);
+    }
+    return addr[dev];
+}
+
+int num_sms() {
+    static int sms[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
+    if (!sms[dev]) {
+        int v = 0;
+        cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
+        sms[dev] = v > 0 ? v : 1;
+    }
+    return sms[dev];
+}
+
+// ---------------------------------------------------------------------------
+// Kernel trace: host-thread-local list of (name, start event, stop event).
+struct TraceRec {
+    const char *name;
+    cudaEvent_t start, stop;
+};
+struct Trace {
+    bool on = false;
+    int max_records = 0;
+    int count = 0;
+    std::vector<TraceRec> recs;  // event pool, reused across enables
+};
+static thread_local Trace g_trace;
+
+void trace_before(cudaStream_t s, const char *kernel_name) {
+    Trace &t = g_trace;
+    if (!t.on || t.count >= t.max_records) return;
+    TraceRec &r = t.recs[t.count];
+    r.name = kernel_name;
+    cudaEventRecord(r.start, s);
+}
+
+void trace_after(cudaStream_t s) {
+    Trace &t = g_trace;
+    if (!t.on || t.count >= t.max_records) return;
+    cudaEventRecord(t.recs[t.count].stop, s);
+    t.count++;
+}
+
+}  // namespace vmoe
+
+using namespace vmoe;
+
+static int capacity_of(const vmoe_problem *p) {
+    if (p->capacity > 0) return p->capacity;
+    double c = ceil(p->capacity_factor * (double)p->k * (double)p->N / (double)p->E);
+    if (c < 1.0) c = 1.0;
+    if (c > (double)p->N) c = (double)p->N;
+    return (int)c;
+}
+
+// Checks the problem statement; fills `d`.  Returns VMOE_OK or an error.
+static int check_problem(const vmoe_problem *p, Dims *d) {
+    if (!p) return VMOE_ERR_INVALID;
+    if (p->T < 1 || p->N < 1 || p->E < 1 || p->k < 1 || p->d_model < 1 || p->d_ff < 1)
+        return VMOE_ERR_INVALID;
+    if (p->k > p->E || p->k > 8) return VMOE_ERR_INVALID;
+    if (p->dtype != VMOE_F32 && p->dtype != VMOE_BF16) return VMOE_ERR_INVALID;
+    if (p->capacity < 0) return VMOE_ERR_INVALID;
+    if (p->capacity == 0 && !(p->capacity_factor > 0.0 && isfinite(p->capacity_factor)))
+        return VMOE_ERR_INVALID;
+    if (p->flags & ~(uint32_t)(VMOE_LOGITS_IN | VMOE_NO_RENORM | VMOE_GELU_TANH))
+        return VMOE_ERR_INVALID;
+    if (p->E > 256) return VMOE_ERR_UNSUPPORTED;
+    if ((long long)p->T * p->E > 1024) return VMOE_ERR_UNSUPPORTED;
+    if (p->d_model % 8 != 0) return VMOE_ERR_UNSUPPORTED;
+    // 32-bit element offsets inside one group / one task are assumed.
+    if ((long long)p->N * p->d_model >= (1LL << 31)) return VMOE_ERR_UNSUPPORTED;
+    if ((long long)p->d_model * p->d_ff >= (1LL << 31)) return VMOE_ERR_UNSUPPORTED;
+    int C = capacity_of(p);
+    if ((long long)C * p->d_ff >= (1LL << 31)) return VMOE_ERR_UNSUPPORTED;
+    d->T = p->T;
+    d->N = p->N;
+    d->d = p->d_model;
+    d->f = p->d_ff;
+    d->E = p->E;
+    d->k = p->k;
+    d->C = C;
+    d->flags = p->flags;
+    d->bf16 = p->dtype == VMOE_BF16;
+    return VMOE_OK;
+}
+
+static bool aligned16(const void *ptr) { return ((uintptr_t)ptr & 15u) == 0; }
+static bool dev_ok(const void *ptr) { return ptr != nullptr && aligned16(ptr); }
+static bool opt_ok(const void *ptr) { return ptr == nullptr || aligned16(ptr); }
+
+static int check_expert_shape(const Dims &d) {
+    if (d.bf16 && (d.d % 128 != 0 || d.f % 128 != 0)) return VMOE_ERR_UNSUPPORTED;
+    if (!d.bf16 && (d.d % 4 != 0 || d.f % 4 != 0)) return VMOE_ERR_UNSUPPORTED;
+    return VMOE_OK;
+}
+
+extern "C" {
+
+int vmoe_version(void) { return VMOE_VERSION; }
+
+const char *vmoe_status_string(int status) {
+    switch (status) {
+        case VMOE_OK: return "VMOE_OK";
+        case VMOE_ERR_INVALID: return "VMOE_ERR_INVALID: invalid argument";
+        case VMOE_ERR_UNSUPPORTED: return "VMOE_ERR_UNSUPPORTED: unsupported shape";
+        case VMOE_ERR_CUDA: return "VMOE_ERR_CUDA: CUDA runtime error";
+        case VMOE_ERR_DEVICE_TIMEOUT: return "VMOE_ERR_DEVICE_TIMEOUT: a kernel gave up a bounded wait";
+        default: return "unknown vmoe status";
+    }
+}
+
+int vmoe_problem_capacity(const vmoe_problem *p) {
+    Dims d;
+    int st = check_problem(p, &d);
+    return st == VMOE_OK ? d.C : st;
+}
+
+int vmoe_route(const vmoe_problem *p, const void *x, const float *w_router,
+               const float *logit_bias, float *logits, int32_t *expert_idx, float *gate,
+               int32_t *slot, int32_t *load, void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    bool given = (p->flags & VMOE_LOGITS_IN) != 0;
+    if (!given && (!dev_ok(x) || !dev_ok(w_router))) return VMOE_ERR_INVALID;
+    if (!opt_ok(logit_bias) || !dev_ok(logits) || !dev_ok(expert_idx) || !dev_ok(gate) ||
+        !dev_ok(slot) || !dev_ok(load))
+        return VMOE_ERR_INVALID;
+    return launch_route(d, given ? nullptr : x, w_router, logit_bias, logits, expert_idx, gate,
+                        slot, load, (cudaStream_t)cuda_stream);
+}
+
+int vmoe_dispatch(const vmoe_problem *p, const void *src, const float *weight,
+                  const int32_t *expert_idx, const int32_t *slot, const int32_t *load,
+                  void *dst, void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    if (!dev_ok(src) || !opt_ok(weight) || !dev_ok(expert_idx) || !dev_ok(slot) ||
+        !dev_ok(load) || !dev_ok(dst))
+        return VMOE_ERR_INVALID;
+    return launch_dispatch(d, src, weight, expert_idx, slot, load, dst, (cudaStream_t)cuda_stream);
+}
+
+int vmoe_combine(const vmoe_problem *p, const void *src, const float *weight,
+                 const int32_t *expert_idx, const int32_t *slot, void *dst, void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    if (!dev_ok(src) || !opt_ok(weight) || !dev_ok(expert_idx) || !dev_ok(slot) || !dev_ok(dst))
+        return VMOE_ERR_INVALID;
+    return launch_combine(d, src, weight, expert_idx, slot, dst, (cudaStream_t)cuda_stream);
+}
+
+int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const void *w2,
+                    const int32_t *load, void *h, void *a, void *ye, void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    if ((st = check_expert_shape(d)) != VMOE_OK) return st;
+    if (!dev_ok(xe) || !dev_ok(w1) || !dev_ok(w2) || !dev_ok(load) || !dev_ok(h) ||
+        !dev_ok(a) || !dev_ok(ye))
+        return VMOE_ERR_INVALID;
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    if (d.bf16)
+        return launch_expert_fwd_bf16(
+            d, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)w1, (const __nv_bfloat16 *)w2,
+            load, (__nv_bfloat16 *)h, (__nv_bfloat16 *)a, (__nv_bfloat16 *)ye, s);
+    return launch_expert_fwd_f32(d, (const float *)xe, (const float *)w1, (const float *)w2, load,
+                                 (float *)h, (float *)a, (float *)ye, s);
+}
+
+size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p) {
+    Dims d;
+    if (check_problem(p, &d) != VMOE_OK) return 0;
+    size_t elem = d.bf16 ? 2 : 4;
+    return (size_t)d.T * d.E * d.C * d.f * elem;
+}
+
+int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,
+                    const void *w1, const void *w2, const void *dye, const int32_t *load,
+                    void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,
+                    void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    if ((st = check_expert_shape(d)) != VMOE_OK) return st;
+    if (!dev_ok(xe) || !dev_ok(h) || !dev_ok(a) || !dev_ok(w1) || !dev_ok(w2) || !dev_ok(dye) ||
+        !dev_ok(load) || !dev_ok(dxe) || !dev_ok(dw1) || !dev_ok(dw2) || !dev_ok(workspace))
+        return VMOE_ERR_INVALID;
+    if (workspace_bytes < vmoe_expert_bwd_workspace_size(p)) return VMOE_ERR_INVALID;
+    cudaStream_t s = (cudaStream_t)cuda_stream;
+    if (d.bf16)
+        return launch_expert_bwd_bf16(
+            d, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)h, (const __nv_bfloat16 *)a,
+            (const __nv_bfloat16 *)w1, (const __nv_bfloat16 *)w2, (const __nv_bfloat16 *)dye, load,
+            (__nv_bfloat16 *)dxe, (__nv_bfloat16 *)dw1, (__nv_bfloat16 *)dw2,
+            (__nv_bfloat16 *)workspace, s);
+    return launch_expert_bwd_f32(d, (const float *)xe, (const float *)h, (const float *)a,
+                                 (const float *)w1, (const float *)w2, (const float *)dye, load,
+                                 (float *)dxe, (float *)dw1, (float *)dw2, (float *)workspace, s);
+}
+
+int vmoe_device_status(int reset) {
+    if (cudaDeviceSynchronize() != cudaSuccess) return VMOE_ERR_CUDA;
+    int *addr = device_status_word();
+    if (!addr) return VMOE_ERR_CUDA;
+    int v = 0;
+    if (cudaMemcpy(&v, addr, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+        return VMOE_ERR_CUDA;
+    if (reset) {
+        int z = 0;
+        if (cudaMemcpy(addr, &z, sizeof(int), cudaMemcpyHostToDevice) != cudaSuccess)
+            return VMOE_ERR_CUDA;
+    }
+    return v;
+}
+
+int vmoe_trace_enable(int max_records) {
+    if (max_records < 1 || max_records > (1 << 20)) return VMOE_ERR_INVALID;
+    Trace &t = g_trace;
+    while ((int)t.recs.size() < max_records) {
+        TraceRec r;
+        r.name = nullptr;
+        if (cudaEventCreate(&r.start) != cudaSuccess) return VMOE_ERR_CUDA;
+        if (cudaEventCreate(&r.stop) != cudaSuccess) {
+            cudaEventDestroy(r.start);
+            return VMOE_ERR_CUDA;
+        }
+        t.recs.push_back(r);
+    }
+    t.max_records = max_records;
+    t.count = 0;
+    t.on = true;
+    return VMOE_OK;
+}
+
+int vmoe_trace_disable(void) {
+    g_trace.on = false;
+    return g_trace.count;
+}
+
+int vmoe_trace_get(int i, const char **kernel_name, float *ms) {
+    Trace &t = g_trace;
+    if (i < 0 || i >= t.count || !kernel_name || !ms) return VMOE_ERR_INVALID;
+    if (cudaEventSynchronize(t.recs[i].stop) != cudaSuccess) return VMOE_ERR_CUDA;
+    if (cudaEventElapsedTime(ms, t.recs[i].start, t.recs[i].stop) != cudaSuccess)
+        return VMOE_ERR_CUDA;
+    *kernel_name = t.recs[i].name;
+    return VMOE_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,103 @@
+// common.cuh -- shared declarations of the libvmoe CUDA sources (internal).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "vmoe.h"
+
+namespace vmoe {
+
+// Validated problem sizes, as the kernels see them.
+struct Dims {
+    int T, N, d, f, E, k, C;
+    unsigned flags;
+    bool bf16;
+    int G() const { return T * E; }
+};
+
+// Host-side hooks (abi.cu).
+void trace_before(cudaStream_t s, const char *kernel_name);
+void trace_after(cudaStream_t s);
+int *device_status_word();  // device address of the current device's status word, or NULL
+int num_sms();              // SM count of the current device
+
+// Returns VMOE_OK or VMOE_ERR_CUDA after a launch.
+inline int launch_result() {
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? VMOE_OK : VMOE_ERR_CUDA;
+}
+
+// Launchers (one file each).
+int launch_route(const Dims &p, const void *x, const float *w_router, const float *bias,
+                 float *logits, int32_t *idx, float *gate, int32_t *slot, int32_t *load,
+                 cudaStream_t s);
+int launch_dispatch(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+                    const int32_t *slot, const int32_t *load, void *dst, cudaStream_t s);
+int launch_combine(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+                   const int32_t *slot, void *dst, cudaStream_t s);
+int launch_expert_fwd_f32(const Dims &p, const float *xe, const float *w1, const float *w2,
+                          const int32_t *load, float *h, float *a, float *ye, cudaStream_t s);
+int launch_expert_bwd_f32(const Dims &p, const float *xe, const float *h, const float *a,
+                          const float *w1, const float *w2, const float *dye,
+                          const int32_t *load, float *dxe, float *dw1, float *dw2, float *dh,
+                          cudaStream_t s);
+int launch_expert_fwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bfloat16 *w1,
+                           const __nv_bfloat16 *w2, const int32_t *load, __nv_bfloat16 *h,
+                           __nv_bfloat16 *a, __nv_bfloat16 *ye, cudaStream_t s);
+int launch_expert_bwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bfloat16 *h,
+                           const __nv_bfloat16 *a, const __nv_bfloat16 *w1,
+                           const __nv_bfloat16 *w2, const __nv_bfloat16 *dye,
+                           const int32_t *load, __nv_bfloat16 *dxe, __nv_bfloat16 *dw1,
+                           __nv_bfloat16 *dw2, __nv_bfloat16 *dh, cudaStream_t s);
+
+// ---------------------------------------------------------------------------
+// Device helpers.
+
+// 8 bf16 <-> 8 floats through one 16-byte vector.
+__device__ __forceinline__ void bf16x8_to_f32(const uint4 &v, float *out) {
+    const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        float2 f = __bfloat1622float2(h[i]);
+        out[2 * i] = f.x;
+        out[2 * i + 1] = f.y;
+    }
+}
+
+__device__ __forceinline__ uint4 f32_to_bf16x8(const float *in) {
+    uint4 v;
+    __nv_bfloat162 *h = reinterpret_cast<__nv_bfloat162 *>(&v);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(in[2 * i], in[2 * i + 1]);
+    return v;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t *>(&h);
+}
+
+// GELU and its derivative: exact erf form by default, tanh form with
+// VMOE_GELU_TANH.  Both call CUDA's erff / expf / tanhf.
+__device__ __forceinline__ float gelu_f(float h, bool tanh_form) {
+    if (tanh_form) {
+        const float c = 0.7978845608028654f;  // sqrt(2/pi)
+        return 0.5f * h * (1.0f + tanhf(c * (h + 0.044715f * h * h * h)));
+    }
+    return 0.5f * h * (1.0f + erff(h * 0.7071067811865476f));
+}
+
+__device__ __forceinline__ float gelu_deriv_f(float h, bool tanh_form) {
+    if (tanh_form) {
+        const float c = 0.7978845608028654f;
+        float th = tanhf(c * (h + 0.044715f * h * h * h));
+        return 0.5f * (1.0f + th) +
+               0.5f * h * (1.0f - th * th) * c * (1.0f + 3.0f * 0.044715f * h * h);
+    }
+    const float inv_sqrt_2pi = 0.3989422804014327f;
+    return 0.5f * (1.0f + erff(h * 0.7071067811865476f)) + h * inv_sqrt_2pi * expf(-0.5f * h * h);
+}
+
+}  // namespace vmoe

@@ -1,0 +1,702 @@
+// gemm_tc.cuh -- K3/K4/K6-K9: the bf16 grouped GEMM of the expert FFN on the
+// sm_103a tensor cores (tcgen05 + TMEM + TMA), one persistent launch over all
+// T*E (task, expert) groups of the merged expert pool.
+//
+// Structure (one CTA per SM, 320 threads):
+//   warp 0      TMA producer: one thread streams 128x64 A tiles and 64xBN B
+//               tiles into a STAGES-deep ring of shared-memory slots
+//               (128-byte swizzle), signalling `full[s]` with the byte count.
+//   warp 1      MMA issuer: one thread issues tcgen05.mma (M=128, N=BN,
+//               K=16, bf16 in, fp32 accumulate in TMEM), commits each slot
+//               back to `empty[s]` and each finished tile to `tmem_full[a]`.
+//               The whole warp zeroes the K-tail rows of weight-gradient tiles.
+//   warps 2-9   epilogue: tcgen05.ld of the accumulator (one TMEM lane per
+//               thread = one output row; two warps per lane quarter split the
+//               columns), the fused elementwise step (GELU, or GELU' of an H
+//               prefetched into registers one chunk ahead), bf16 packing, a
+//               per-warp staging tile in shared memory and coalesced 16-byte
+//               row stores.  The accumulator is double buffered in TMEM
+//               (2 x BN columns), so tile i's epilogue overlaps tile i+1's
+//               main loop.
+// Tiles are distributed statically: CTA b takes tiles b, b + grid, ...  In
+// row mode (H = Xe W1 etc.) a group contributes ceil(load/128) x N/BN tiles,
+// counted from the device-resident loads by every CTA with a block scan, so
+// empty groups cost nothing and no host round trip is needed.  In weight-
+// gradient mode (dW1 = Xe^T dH etc.) every group contributes (M/128) x (N/BN)
+// tiles whose K = load[g] rows; an empty group's tile is written as zeros.
+//
+// Every wait on an mbarrier is bounded in time; a wait that runs out sets the
+// library's device status word to VMOE_ERR_DEVICE_TIMEOUT and an abort flag
+// that the other roles see, and the CTA drains its copies and MMAs in flight
+// and frees its TMEM before it returns.
+#pragma once
+
+#include <cuda.h>  // CUtensorMap and its enums (types only; the encoder is fetched at run time)
+
+#include "common.cuh"
+
+namespace vmoe {
+namespace tc {
+
+constexpr int BM = 128;  // rows of one MMA tile (TMEM lanes)
+constexpr int BK = 64;   // K per pipeline slot = one 128-byte swizzle row of bf16
+constexpr int THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
+constexpr int EPI_WARP_BYTES = 32 * 80;  // 32 rows x (64 data + 16 pad) bytes
+constexpr int MAX_G = 1024;
+constexpr unsigned long long TIMEOUT_NS = 4000000000ull;
+
+enum { MODE_ROW = 0, MODE_WGRAD = 1 };
+enum { EPI_STORE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
+
+template <int BN>
+struct Shape {
+    static constexpr int STAGES = BN == 256 ? 4 : 6;
+    static constexpr uint32_t A_BYTES = BM * BK * 2;
+    static constexpr uint32_t B_BYTES = BN * BK * 2;
+    static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr uint32_t TMEM_COLS = 2 * BN;
+    static constexpr int NUM_BARS = 2 * STAGES + 5;
+    static constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * STAGE_BYTES + 8 * EPI_WARP_BYTES +
+                                         NUM_BARS * 8 + 16 + THREADS * 4 + (MAX_G + 1) * 4;
+};
+
+struct Args {
+    int G, C;
+    int N;        // output columns
+    int K_fixed;  // row mode: reduction length
+    int M_fixed;  // weight-gradient mode: output rows
+    int tiles_n;  // N / BN
+    int tiles_m;  // weight-gradient mode: M_fixed / BM; row mode: ceil(C / BM)
+    const int32_t *load;
+    __nv_bfloat16 *D;          // output
+    __nv_bfloat16 *D2;         // EPI_GELU: A = GELU(H)
+    const __nv_bfloat16 *aux;  // EPI_DGELU: H
+    long long sD;              // group stride of D / D2 / aux (elements)
+    int ldd;                   // row stride of D / D2 / aux (elements)
+    int gelu_tanh;
+    int *status;
+};
+
+// ---------------------------------------------------------------------------
+// PTX wrappers.
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}\n"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+// Bounded wait for the phase of parity `parity` of barrier `bar`.
+static __device__ __noinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort_flag,
+                                        int *status) {
+    if (mbar_try_wait(bar, parity)) return true;
+    const unsigned long long t0 = global_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(bar, parity)) return true;
+        if ((i & 63u) == 0) {
+            if (*abort_flag) return false;
+            if (global_ns() - t0 > TIMEOUT_NS) {
+                *abort_flag = 1;
+                if (status) atomicExch(status, (int)VMOE_ERR_DEVICE_TIMEOUT);
+                return false;
+            }
+        }
+    }
+}
+__device__ __forceinline__ void fence_barrier_init() {
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
+                                            int c0, int c1, int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+__device__ __forceinline__ void prefetch_map(const CUtensorMap *map) {
+    asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
+}
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols) {
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem),
+                 "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}\n" ::"r"(tmem_d),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     bar)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+        "%12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, "
+        "%30, %31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]),
+          "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]),
+          "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle (tcgen05 format: start
+// address, leading and stride byte offsets in 16-byte units, version 1 at bit
+// 46, layout SWIZZLE_128B = 2 at bits 61-63).
+__device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+// Operand tiles in shared memory:
+//  K-major (K contiguous):  rows of 64 K-elements = 128 bytes, 8-row swizzle
+//    atoms of 1024 bytes stacked along M/N (SBO = 1024).  Step k16 -> +32 bytes.
+//  MN-major (M/N contiguous): chunks of 64 MN-elements x 64 K-rows (8 KiB),
+//    one TMA box each, stacked along M/N (LBO = 8192, the MN chunk stride);
+//    8-row K groups are 1024 bytes apart (SBO).  Step k16 -> +2048 bytes.
+__device__ __forceinline__ uint64_t operand_desc(uint32_t tile, int kk, bool mn_major) {
+    return mn_major ? sdesc_sw128(tile + kk * 2048, 8192, 1024)
+                    : sdesc_sw128(tile + kk * 32, 16, 1024);
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
+// A and B bf16 (bits 7-9, 10-12 = 1), A / B MN-major (bits 15 / 16),
+// N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+__host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn, bool b_mn) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((a_mn ? 1u : 0u) << 15) |
+           ((b_mn ? 1u : 0u) << 16) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+struct Tile {
+    int g, m_blk, n_blk, kblocks, kvalid, rows_valid;
+};
+
+template <int MODE>
+__device__ __forceinline__ Tile decode_tile(const Args &a, const int *prefix, int u) {
+    Tile t;
+    if (MODE == MODE_ROW) {
+        int lo = 0, hi = a.G;  // prefix[lo] <= u < prefix[hi]
+        while (hi - lo > 1) {
+            int mid = (lo + hi) >> 1;
+            if (prefix[mid] <= u) lo = mid; else hi = mid;
+        }
+        t.g = lo;
+        int local = u - prefix[lo];
+        t.m_blk = local / a.tiles_n;
+        t.n_blk = local - t.m_blk * a.tiles_n;
+        t.kblocks = a.K_fixed / BK;
+        t.kvalid = a.K_fixed;
+        int L = __ldg(a.load + t.g);
+        t.rows_valid = L < 0 ? 0 : (L > a.C ? a.C : L);
+    } else {
+        int tpg = a.tiles_m * a.tiles_n;
+        t.g = u / tpg;
+        int local = u - t.g * tpg;
+        t.m_blk = local / a.tiles_n;
+        t.n_blk = local - t.m_blk * a.tiles_n;
+        int L = __ldg(a.load + t.g);
+        L = L < 0 ? 0 : (L > a.C ? a.C : L);
+        t.kvalid = L;
+        t.kblocks = (L + BK - 1) / BK;
+        t.rows_valid = a.M_fixed;
+    }
+    return t;
+}
+
+template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
+__global__ void __launch_bounds__(THREADS, 1)
+grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                    Args args) {
+    using S = Shape<BN>;
+    constexpr int STAGES = S::STAGES;
+    constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
+
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+    const uint32_t tiles_addr = smem_u32(smem);
+    uint8_t *epi_base = smem + STAGES * S::STAGE_BYTES;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + 8 * EPI_WARP_BYTES);
+    int *misc = reinterpret_cast<int *>(bars + S::NUM_BARS);  // [0] tmem base, [1] abort, [2] total
+    int *scan_tmp = misc + 4;
+    int *prefix = scan_tmp + THREADS;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    auto bar_full = [&](int s) { return smem_u32(bars + s); };
+    auto bar_empty = [&](int s) { return smem_u32(bars + STAGES + s); };
+    auto bar_tfull = [&](int a) { return smem_u32(bars + 2 * STAGES + a); };
+    auto bar_tempty = [&](int a) { return smem_u32(bars + 2 * STAGES + 2 + a); };
+    const uint32_t bar_drain = smem_u32(bars + 2 * STAGES + 4);
+    volatile int *abort_flag = misc + 1;
+
+    if (tid == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(bar_full(s), 1);
+            mbar_init(bar_empty(s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(bar_tfull(a), 1);
+            mbar_init(bar_tempty(a), 8);
+        }
+        mbar_init(bar_drain, 1);
+        misc[1] = 0;
+        fence_barrier_init();
+        fence_proxy_async();
+        prefetch_map(&tmA);
+        prefetch_map(&tmB);
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(misc), S::TMEM_COLS);
+        tmem_relinquish();
+    }
+
+    // Tile count (and, in row mode, the per-group tile prefix).
+    int total;
+    if (MODE == MODE_ROW) {
+        const int G = args.G;
+        const int per = (G + THREADS - 1) / THREADS;
+        const int g0 = min(G, tid * per), g1 = min(G, g0 + per);
+        int local = 0;
+        for (int g = g0; g < g1; ++g) {
+            int L = __ldg(args.load + g);
+            L = L < 0 ? 0 : (L > args.C ? args.C : L);
+            local += ((L + BM - 1) / BM) * args.tiles_n;
+        }
+        scan_tmp[tid] = local;
+        __syncthreads();
+        if (warp == 0) {  // exclusive scan of THREADS partials, THREADS/32 per lane
+            constexpr int PER = THREADS / 32;
+            int v[PER], s = 0;
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                v[i] = scan_tmp[lane * PER + i];
+                s += v[i];
+            }
+            int incl = s;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                int y = __shfl_up_sync(0xffffffffu, incl, o);
+                if (lane >= o) incl += y;
+            }
+            int run = incl - s;
+#pragma unroll
+            for (int i = 0; i < PER; ++i) {
+                scan_tmp[lane * PER + i] = run;
+                run += v[i];
+            }
+            if (lane == 31) misc[2] = incl;
+        }
+        __syncthreads();
+        int run = scan_tmp[tid];
+        for (int g = g0; g < g1; ++g) {
+            prefix[g] = run;
+            int L = __ldg(args.load + g);
+            L = L < 0 ? 0 : (L > args.C ? args.C : L);
+            run += ((L + BM - 1) / BM) * args.tiles_n;
+        }
+        if (tid == 0) prefix[G] = misc[2];
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    total = (MODE == MODE_ROW) ? misc[2] : args.G * args.tiles_m * args.tiles_n;
+    const uint32_t tmem_base = (uint32_t)misc[0];
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            int stage = 0;
+            uint32_t phase = 0;
+            int issued[STAGES];
+#pragma unroll
+            for (int s = 0; s < STAGES; ++s) issued[s] = 0;
+            bool ok = true;
+            for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+                const Tile t = decode_tile<MODE>(args, prefix, u);
+                for (int kb = 0; kb < t.kblocks; ++kb) {
+                    if (!wait_phase(bar_empty(stage), phase ^ 1u, abort_flag, args.status)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t sa = tiles_addr + stage * S::STAGE_BYTES;
+                    const uint32_t sb = sa + S::A_BYTES;
+                    const uint32_t fb = bar_full(stage);
+                    mbar_expect_tx(fb, S::STAGE_BYTES);
+                    if (MODE == MODE_ROW) {
+                        tma_load_3d(sa, &tmA, fb, kb * BK, t.m_blk * BM, t.g);
+                        if (B_MN) {
+#pragma unroll
+                            for (int c = 0; c < BN / 64; ++c)
+                                tma_load_3d(sb + c * 8192, &tmB, fb, t.n_blk * BN + c * 64, kb * BK, t.g);
+                        } else {
+                            tma_load_3d(sb, &tmB, fb, kb * BK, t.n_blk * BN, t.g);
+                        }
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < BM / 64; ++c)
+                            tma_load_3d(sa + c * 8192, &tmA, fb, t.m_blk * BM + c * 64, kb * BK, t.g);
+#pragma unroll
+                        for (int c = 0; c < BN / 64; ++c)
+                            tma_load_3d(sb + c * 8192, &tmB, fb, t.n_blk * BN + c * 64, kb * BK, t.g);
+                    }
+                    issued[stage]++;
+                    if (++stage == STAGES) {
+                        stage = 0;
+                        phase ^= 1u;
+                    }
+                }
+            }
+            if (*abort_flag) {  // let copies in flight land before the CTA exits
+                int dummy = 0;
+                for (int s = 0; s < STAGES; ++s)
+                    if (issued[s] > 0) {
+                        const unsigned long long t0 = global_ns();
+                        while (!mbar_try_wait(bar_full(s), (uint32_t)((issued[s] - 1) & 1)) &&
+                               global_ns() - t0 < 100000000ull)
+                            ++dummy;
+                    }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        int stage = 0;
+        uint32_t phase = 0;
+        int it = 0;
+        bool ok = true;
+        for (int u = blockIdx.x; u < total && ok; u += gridDim.x, ++it) {
+            const Tile t = decode_tile<MODE>(args, prefix, u);
+            const int acc = it & 1;
+            const uint32_t aph = (uint32_t)((it >> 1) & 1);
+            if (!wait_phase(bar_tempty(acc), aph ^ 1u, abort_flag, args.status)) break;
+            tc_fence_after();
+            const uint32_t dtmem = tmem_base + (uint32_t)(acc * BN);
+            if (t.kblocks == 0) {
+                if (lane == 0) mbar_arrive(bar_tfull(acc));
+                __syncwarp();
+                continue;
+            }
+            for (int kb = 0; kb < t.kblocks; ++kb) {
+                if (!wait_phase(bar_full(stage), phase, abort_flag, args.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t sa = tiles_addr + stage * S::STAGE_BYTES;
+                const uint32_t sb = sa + S::A_BYTES;
+                int nk = BK / 16;
+                if (MODE == MODE_WGRAD && kb == t.kblocks - 1) {
+                    // K tail: the MMA reads rows [0, 16*nk) of the slot; rows
+                    // [rem, 16*nk) lie past this group's load and are zeroed in
+                    // both operands (one 128-byte line per K row per 64-wide chunk).
+                    const int rem = t.kvalid - kb * BK;
+                    nk = (rem + 15) >> 4;
+                    const int z0 = rem, z1 = nk * 16;
+                    if (z0 < z1) {
+                        const int rows = z1 - z0;
+                        constexpr int CH = BM / 64 + BN / 64;
+                        const int units = CH * rows * 8;
+                        uint8_t *slot_ptr = smem + stage * S::STAGE_BYTES;
+                        for (int i = lane; i < units; i += 32) {
+                            int c = i / (rows * 8);
+                            int w = i - c * rows * 8;
+                            int r = z0 + (w >> 3);
+                            int q = w & 7;
+                            uint8_t *base = (c < BM / 64) ? slot_ptr + c * 8192
+                                                          : slot_ptr + S::A_BYTES + (c - BM / 64) * 8192;
+                            *reinterpret_cast<uint4 *>(base + r * 128 + q * 16) = make_uint4(0, 0, 0, 0);
+                        }
+                        fence_proxy_async();
+                    }
+                    __syncwarp();
+                }
+                if (lane == 0) {
+                    for (int kk = 0; kk < nk; ++kk)
+                        mma_bf16(dtmem, operand_desc(sa, kk, A_MN), operand_desc(sb, kk, B_MN), IDESC,
+                                 (kb | kk) != 0 ? 1u : 0u);
+                    mma_commit(bar_empty(stage));
+                }
+                __syncwarp();
+                if (++stage == STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            if (lane == 0) mma_commit(bar_tfull(acc));
+            __syncwarp();
+        }
+        if (lane == 0) {  // all MMAs of this CTA complete before TMEM is freed
+            mma_commit(bar_drain);
+            const unsigned long long t0 = global_ns();
+            while (!mbar_try_wait(bar_drain, 0) && global_ns() - t0 < 1000000000ull) {
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        // Warps 2..9.  Warps w and w+4 share TMEM lane quarter q = w & 3 (rows
+        // 32q..32q+31 of the tile) and split its BN columns in halves; each
+        // thread owns one row and works through its half in 32-column chunks.
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int half = ew >> 2;
+        constexpr int COLS = BN / 2;
+        constexpr int NCH = COLS / 32;
+        uint8_t *stg = epi_base + ew * EPI_WARP_BYTES;
+        const bool tanh_form = args.gelu_tanh != 0;
+        const int sub_r = lane >> 2, sub_c = lane & 3;  // row-store mapping: 8 rows x 4 x 16 B
+        // EPI_DGELU: the H values of this thread's row for the current chunk,
+        // loaded one chunk ahead (and across tiles) so the epilogue never waits
+        // on a fresh global load.
+        uint4 hcur[4], hnxt[4];
+        auto load_h = [&](const Tile &tl, int c, uint4 (&dst)[4]) {
+            const int r0 = tl.m_blk * BM + q * 32;
+            if (r0 + lane < tl.rows_valid) {
+                const uint4 *src = reinterpret_cast<const uint4 *>(
+                    args.aux + (long long)tl.g * args.sD + (long long)(r0 + lane) * args.ldd +
+                    tl.n_blk * BN + half * COLS + c * 32);
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
+            } else {
+#pragma unroll
+                for (int i = 0; i < 4; ++i) dst[i] = make_uint4(0, 0, 0, 0);
+            }
+        };
+        // Stage 32 packed rows of this warp and store them coalesced, masked to
+        // the valid rows.
+        auto store_rows = [&](__nv_bfloat16 *base, int nvalid) {
+            __syncwarp();
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = i * 8 + sub_r;
+                if (r < nvalid)
+                    *reinterpret_cast<uint4 *>(base + (long long)r * args.ldd + sub_c * 8) =
+                        *reinterpret_cast<const uint4 *>(stg + r * 80 + sub_c * 16);
+            }
+            __syncwarp();
+        };
+        int it = 0;
+        Tile t = decode_tile<MODE>(args, prefix, blockIdx.x < total ? blockIdx.x : 0);
+        if (EPI == EPI_DGELU && blockIdx.x < total) load_h(t, 0, hcur);
+        for (int u = blockIdx.x; u < total; u += gridDim.x, ++it) {
+            const bool have_next = u + (int)gridDim.x < total;
+            const Tile tn = decode_tile<MODE>(args, prefix, have_next ? u + gridDim.x : u);
+            const int acc = it & 1;
+            const uint32_t aph = (uint32_t)((it >> 1) & 1);
+            if (!wait_phase(bar_tfull(acc), aph, abort_flag, args.status)) break;
+            tc_fence_after();
+            const int row0 = t.m_blk * BM + q * 32;  // this warp's first row in the group
+            int nvalid = t.rows_valid - row0;
+            nvalid = nvalid < 0 ? 0 : (nvalid > 32 ? 32 : nvalid);
+            const long long gofs = (long long)t.g * args.sD + (long long)row0 * args.ldd +
+                                   t.n_blk * BN + half * COLS;
+            const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
+                                  (uint32_t)(acc * BN + half * COLS);
+            for (int c = 0; c < NCH; ++c) {
+                if (EPI == EPI_DGELU) {
+                    if (c + 1 < NCH) load_h(t, c + 1, hnxt);
+                    else if (have_next) load_h(tn, 0, hnxt);
+                }
+                if (nvalid > 0) {
+                    float v[32];
+                    if (t.kblocks > 0) {
+                        uint32_t r[32];
+                        tmem_ld32(trow + c * 32, r);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                    } else {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                    }
+                    if (EPI == EPI_DGELU) {
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            float hv[8];
+                            bf16x8_to_f32(hcur[i], hv);
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_f(hv[e], tanh_form);
+                        }
+                    }
+#pragma unroll
+                    for (int i = 0; i < 4; ++i)
+                        *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(v + i * 8);
+                    store_rows(args.D + gofs + c * 32, nvalid);
+                    if (EPI == EPI_GELU) {
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            float gv[8];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) gv[e] = gelu_f(v[i * 8 + e], tanh_form);
+                            *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(gv);
+                        }
+                        store_rows(args.D2 + gofs + c * 32, nvalid);
+                    }
+                }
+                if (EPI == EPI_DGELU) {
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) hcur[i] = hnxt[i];
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_tempty(acc));
+            t = tn;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem_base, S::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
+// Host side.
+
+// Encodes a rank-3 bf16 tensor map {inner, mid, outer} (inner contiguous) with
+// a {64, box_mid, 1} box and 128-byte swizzle; out-of-range elements read 0.
+bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, uint64_t outer,
+              uint32_t box_mid);
+
+template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
+int launch(const CUtensorMap &ma, const CUtensorMap &mb, const Args &a, long long max_tiles,
+           cudaStream_t s, const char *name) {
+    using S = Shape<BN>;
+    auto kern = grouped_gemm_kernel<BN, MODE, A_MN, B_MN, EPI>;
+    static uint64_t attr_done = 0;  // one bit per device
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 64 && !(attr_done >> dev & 1ull)) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)S::SMEM_BYTES) != cudaSuccess)
+            return VMOE_ERR_CUDA;
+        attr_done |= 1ull << dev;
+    }
+    if (max_tiles <= 0) return VMOE_OK;
+    long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
+    trace_before(s, name);
+    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, a);
+    trace_after(s);
+    return launch_result();
+}
+
+inline Args base_args(const Dims &p, const int32_t *load) {
+    Args a = {};
+    a.G = p.G();
+    a.C = p.C;
+    a.load = load;
+    a.gelu_tanh = (p.flags & VMOE_GELU_TANH) != 0;
+    a.status = device_status_word();
+    return a;
+}
+
+// Row-mode GEMM: D[g][C rows][N] = act[g][C][K] * B, B MN-major ([K][N]) or
+// K-major ([N][K]).
+template <int EPI, bool B_MN>
+int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16 *w, int N,
+                    const int32_t *load, __nv_bfloat16 *D, __nv_bfloat16 *D2,
+                    const __nv_bfloat16 *aux, cudaStream_t s, const char *name) {
+    const int G = p.G(), C = p.C;
+    const bool wide = N % 256 == 0;
+    const int BN = wide ? 256 : 128;
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, act, K, C, G, 128)) return VMOE_ERR_CUDA;
+    bool okb = B_MN ? make_map(&mb, w, N, K, G, 64) : make_map(&mb, w, K, N, G, BN);
+    if (!okb) return VMOE_ERR_CUDA;
+    Args a = base_args(p, load);
+    a.N = N;
+    a.K_fixed = K;
+    a.tiles_n = N / BN;
+    a.tiles_m = (C + BM - 1) / BM;
+    a.D = D;
+    a.D2 = D2;
+    a.aux = aux;
+    a.sD = (long long)C * N;
+    a.ldd = N;
+    long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
+    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, a, max_tiles, s, name)
+                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, a, max_tiles, s, name);
+}
+
+// Weight-gradient GEMM: D[g][M][N] = act1[g][C][M]^T * act2[g][C][N], summed
+// over each group's load[g] rows; both operands MN-major.
+inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __nv_bfloat16 *act2,
+                      int N, const int32_t *load, __nv_bfloat16 *D, cudaStream_t s,
+                      const char *name) {
+    const int G = p.G(), C = p.C;
+    const bool wide = N % 256 == 0;
+    const int BN = wide ? 256 : 128;
+    CUtensorMap ma, mb;
+    if (!make_map(&ma, act1, M, C, G, 64)) return VMOE_ERR_CUDA;
+    if (!make_map(&mb, act2, N, C, G, 64)) return VMOE_ERR_CUDA;
+    Args a = base_args(p, load);
+    a.N = N;
+    a.M_fixed = M;
+    a.tiles_n = N / BN;
+    a.tiles_m = M / BM;
+    a.D = D;
+    a.sD = (long long)M * N;
+    a.ldd = N;
+    long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
+    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, a, max_tiles, s, name)
+                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, a, max_tiles, s, name);
+}
+
+}  // namespace tc
+}  // namespace vmoe

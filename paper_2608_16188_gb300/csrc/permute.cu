@@ -1,0 +1,152 @@
+// permute.cu -- K2 dispatch (token rows -> expert-contiguous [T,E,C,d]
+// buffers) and K5 combine (expert rows -> token order, gate-weighted).
+//
+// Both are pure data movement with one warp per row and 16-byte vectors
+// (d % 8 == 0 for bf16 and fp32 rows alike).  Dispatch is a scatter: warp w
+// < T*N*k copies the kept choice w to its slot; warps past that zero the
+// padding rows s >= load of every group, so every element of dst is written
+// exactly once and no memset is needed.  Combine is the gather form of the
+// scatter-add: one warp per token sums its kept choices in the order
+// j = 0..k-1 in fp32 and writes the row once, with no atomics.
+#include "common.cuh"
+
+namespace vmoe {
+namespace {
+
+constexpr int PM_THREADS = 256;
+constexpr int PM_WARPS = PM_THREADS / 32;
+
+template <typename T>
+struct Vec;
+template <>
+struct Vec<float> {
+    static constexpr int n = 4;
+    __device__ static void load(const uint4 &v, float *o) {
+        o[0] = __uint_as_float(v.x);
+        o[1] = __uint_as_float(v.y);
+        o[2] = __uint_as_float(v.z);
+        o[3] = __uint_as_float(v.w);
+    }
+    __device__ static uint4 store(const float *o) {
+        return make_uint4(__float_as_uint(o[0]), __float_as_uint(o[1]), __float_as_uint(o[2]),
+                          __float_as_uint(o[3]));
+    }
+};
+template <>
+struct Vec<__nv_bfloat16> {
+    static constexpr int n = 8;
+    __device__ static void load(const uint4 &v, float *o) { bf16x8_to_f32(v, o); }
+    __device__ static uint4 store(const float *o) { return f32_to_bf16x8(o); }
+};
+
+template <typename T>
+__global__ void __launch_bounds__(PM_THREADS)
+dispatch_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
+                const int32_t *__restrict__ idx, const int32_t *__restrict__ slot,
+                const int32_t *__restrict__ load, T *__restrict__ dst) {
+    constexpr int V = Vec<T>::n;
+    const long long row = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    const int nvec = p.d / V;
+    const long long n_assign = (long long)p.T * p.N * p.k;
+    if (row < n_assign) {
+        int s = slot[row];
+        if (s < 0) return;
+        long long tn = row / p.k;  // t*N + n
+        int t = (int)(tn / p.N);
+        int e = idx[row];
+        const uint4 *in = reinterpret_cast<const uint4 *>(src + tn * p.d);
+        uint4 *out = reinterpret_cast<uint4 *>(dst + (((long long)t * p.E + e) * p.C + s) * p.d);
+        if (weight == nullptr) {
+            for (int v = lane; v < nvec; v += 32) out[v] = __ldg(in + v);
+        } else {
+            float w = weight[row];
+            for (int v = lane; v < nvec; v += 32) {
+                float f[V];
+                Vec<T>::load(__ldg(in + v), f);
+#pragma unroll
+                for (int q = 0; q < V; ++q) f[q] *= w;
+                out[v] = Vec<T>::store(f);
+            }
+        }
+        return;
+    }
+    long long r = row - n_assign;  // padding candidate: (g, s)
+    if (r >= (long long)p.T * p.E * p.C) return;
+    long long g = r / p.C;
+    int s = (int)(r - g * p.C);
+    if (s < load[g]) return;
+    uint4 *out = reinterpret_cast<uint4 *>(dst + r * p.d);
+    for (int v = lane; v < nvec; v += 32) out[v] = make_uint4(0u, 0u, 0u, 0u);
+}
+
+template <typename T>
+__global__ void __launch_bounds__(PM_THREADS)
+combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
+               const int32_t *__restrict__ idx, const int32_t *__restrict__ slot,
+               T *__restrict__ dst) {
+    constexpr int V = Vec<T>::n;
+    const long long tn = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
+    if (tn >= (long long)p.T * p.N) return;
+    const int lane = threadIdx.x & 31;
+    const int nvec = p.d / V;
+    const int t = (int)(tn / p.N);
+    int ej[8], sj[8];
+    float wj[8];
+    for (int j = 0; j < p.k; ++j) {
+        ej[j] = idx[tn * p.k + j];
+        sj[j] = slot[tn * p.k + j];
+        wj[j] = weight ? weight[tn * p.k + j] : 1.0f;
+    }
+    uint4 *out = reinterpret_cast<uint4 *>(dst + tn * p.d);
+    for (int v = lane; v < nvec; v += 32) {
+        float acc[V];
+#pragma unroll
+        for (int q = 0; q < V; ++q) acc[q] = 0.0f;
+        for (int j = 0; j < p.k; ++j) {
+            if (sj[j] < 0) continue;
+            const uint4 *in = reinterpret_cast<const uint4 *>(
+                src + (((long long)t * p.E + ej[j]) * p.C + sj[j]) * p.d);
+            float f[V];
+            Vec<T>::load(__ldg(in + v), f);
+#pragma unroll
+            for (int q = 0; q < V; ++q) acc[q] = fmaf(wj[j], f[q], acc[q]);
+        }
+        out[v] = Vec<T>::store(acc);
+    }
+}
+
+}  // namespace
+
+int launch_dispatch(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+                    const int32_t *slot, const int32_t *load, void *dst, cudaStream_t s) {
+    long long rows = (long long)p.T * p.N * p.k + (long long)p.T * p.E * p.C;
+    long long blocks = (rows + PM_WARPS - 1) / PM_WARPS;
+    if (blocks > 0x7fffffffLL) return VMOE_ERR_UNSUPPORTED;
+    trace_before(s, "dispatch");
+    if (p.bf16)
+        dispatch_kernel<__nv_bfloat16><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+            p, (const __nv_bfloat16 *)src, weight, idx, slot, load, (__nv_bfloat16 *)dst);
+    else
+        dispatch_kernel<float><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+            p, (const float *)src, weight, idx, slot, load, (float *)dst);
+    trace_after(s);
+    return launch_result();
+}
+
+int launch_combine(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+                   const int32_t *slot, void *dst, cudaStream_t s) {
+    long long rows = (long long)p.T * p.N;
+    long long blocks = (rows + PM_WARPS - 1) / PM_WARPS;
+    trace_before(s, "combine");
+    if (p.bf16)
+        combine_kernel<__nv_bfloat16><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+            p, (const __nv_bfloat16 *)src, weight, idx, slot, (__nv_bfloat16 *)dst);
+    else
+        combine_kernel<float><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+            p, (const float *)src, weight, idx, slot, (float *)dst);
+    trace_after(s);
+    return launch_result();
+}
+
+}  // namespace vmoe

@@ -1,0 +1,74 @@
+"""Device buffers and the call sequence of one adaptation step (steps a1..a12).
+
+Plumbing only: torch allocates the caller-owned device buffers the C ABI writes
+into, and ``StepRunner`` issues the seven library calls of one step in order on
+one stream.  No arithmetic of the method happens here.
+"""
+from __future__ import annotations
+
+import torch
+
+from . import (VMOE_BF16, vmoe_combine, vmoe_dispatch, vmoe_expert_bwd,
+               vmoe_expert_bwd_workspace_size, vmoe_expert_fwd, vmoe_problem_capacity, vmoe_route)
+
+
+class Buffers:
+    """Every intermediate and output of one step for problem ``p`` on ``device``."""
+
+    def __init__(self, p, device="cuda"):
+        T, N, d, f, E, k = p.T, p.N, p.d_model, p.d_ff, p.E, p.k
+        C = vmoe_problem_capacity(p)
+        dt = torch.bfloat16 if p.dtype == VMOE_BF16 else torch.float32
+        self.C = C
+        self.dtype = dt
+        f32, i32 = torch.float32, torch.int32
+        e = lambda *shape, dtype=dt: torch.empty(shape, dtype=dtype, device=device)  # noqa: E731
+        self.logits = e(T, N, E, dtype=f32)
+        self.idx = e(T, N, k, dtype=i32)
+        self.gate = e(T, N, k, dtype=f32)
+        self.slot = e(T, N, k, dtype=i32)
+        self.load = e(T, E, dtype=i32)
+        self.xe = e(T, E, C, d)
+        self.h = e(T, E, C, f)
+        self.a = e(T, E, C, f)
+        self.ye = e(T, E, C, d)
+        self.y = e(T, N, d)
+        self.dye = e(T, E, C, d)
+        self.dxe = e(T, E, C, d)
+        self.dw1 = e(T, E, d, f)
+        self.dw2 = e(T, E, f, d)
+        self.dx = e(T, N, d)
+        self.workspace = torch.empty(vmoe_expert_bwd_workspace_size(p), dtype=torch.uint8,
+                                     device=device)
+
+
+class StepRunner:
+    """Issues the library calls of one forward + backward step.
+
+    ``inputs`` holds device tensors x, dy [T,N,d], w_router [T,d,E], bias [T,E]
+    or None, w1 [T,E,d,f], w2 [T,E,f,d].
+    """
+
+    def __init__(self, p, inputs, bufs: Buffers | None = None):
+        self.p = p
+        self.inp = inputs
+        self.b = bufs if bufs is not None else Buffers(p, inputs["x"].device)
+
+    def forward(self, stream=None):
+        p, i, b = self.p, self.inp, self.b
+        vmoe_route(p, i["x"], i["w_router"], i.get("bias"), b.logits, b.idx, b.gate, b.slot,
+                   b.load, stream)
+        vmoe_dispatch(p, i["x"], None, b.idx, b.slot, b.load, b.xe, stream)
+        vmoe_expert_fwd(p, b.xe, i["w1"], i["w2"], b.load, b.h, b.a, b.ye, stream)
+        vmoe_combine(p, b.ye, b.gate, b.idx, b.slot, b.y, stream)
+
+    def backward(self, stream=None):
+        p, i, b = self.p, self.inp, self.b
+        vmoe_dispatch(p, i["dy"], b.gate, b.idx, b.slot, b.load, b.dye, stream)
+        vmoe_expert_bwd(p, b.xe, b.h, b.a, i["w1"], i["w2"], b.dye, b.load, b.dxe, b.dw1, b.dw2,
+                        b.workspace, stream=stream)
+        vmoe_combine(p, b.dxe, None, b.idx, b.slot, b.dx, stream)
+
+    def step(self, stream=None):
+        self.forward(stream)
+        self.backward(stream)
