@@ -388,6 +388,9 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=20.0,
                     help="seconds of oracle work for the cpu_baseline sample")
+    ap.add_argument("--tasks", type=int, default=0,
+                    help="run only the first TASKS tasks of the workload (same per-group shapes; "
+                         "used to size profiler captures)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -397,6 +400,8 @@ def main():
     if world != args.gpus and "RANK" in os.environ:
         ap.error("--gpus %d but WORLD_SIZE=%d" % (args.gpus, world))
     cfg = workloads.CONFIGS[args.config]
+    if args.tasks:
+        cfg = cfg.with_(T=min(args.tasks, cfg.T))
     if args.impl == "reference":
         if rank != 0:
             return
