@@ -161,6 +161,29 @@ int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const 
                     void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,
                     void *cuda_stream);
 
+/* Size in bytes of the device array behind vmoe_expert_bwd_static_scratch. */
+#define VMOE_STATIC_SCRATCH_BYTES (64u << 20)
+
+/* vmoe_expert_bwd without a caller-supplied workspace, for callers that cannot
+ * allocate device memory: a plug-in whose host framework owns every device
+ * buffer, or a deployment that allows no device allocation after start-up.
+ * The paper has no counterpart; this is a packaging choice of the library.
+ *   Arguments, layouts and results are those of vmoe_expert_bwd.  The dH
+ *   scratch is a 64 MiB array compiled into the library, which every GPU that
+ *   loads the library holds until the process exits; the call itself allocates
+ *   nothing.  A problem whose vmoe_expert_bwd_workspace_size exceeds
+ *   VMOE_STATIC_SCRATCH_BYTES returns VMOE_ERR_UNSUPPORTED with nothing
+ *   launched.  The first call on a device looks up the array's device address
+ *   (cudaGetSymbolAddress) with that device current; make that first call
+ *   before any stream capture.  Every call on a device shares the one array,
+ *   which keeps whatever the last call left in it, so calls whose kernels
+ *   overlap on the GPU (other streams, other host threads) race and corrupt
+ *   each other's dH; issue them in order on one stream. */
+int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void *xe, const void *h,
+                                   const void *a, const void *w1, const void *w2, const void *dye,
+                                   const int32_t *load, void *dxe, void *dw1, void *dw2,
+                                   void *cuda_stream);
+
 /* Combine back to token order: dst[t,n,:] = sum over kept choices j (slot >= 0)
  * of w * src[t, expert_idx_j, slot_j, :], w = weight[t,n,j] or 1 if NULL,
  * summed in fp32 in the order j = 0..k-1 and rounded once; a token with every

@@ -34,8 +34,8 @@ VMOE_GELU_TANH = 1 << 2
 # Every symbol include/vmoe.h declares.
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
-           "vmoe_expert_bwd", "vmoe_combine", "vmoe_device_status", "vmoe_trace_enable",
-           "vmoe_trace_disable", "vmoe_trace_get")
+           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine",
+           "vmoe_device_status", "vmoe_trace_enable", "vmoe_trace_disable", "vmoe_trace_get")
 
 
 class VmoeError(RuntimeError):
@@ -75,6 +75,7 @@ def library():
             "vmoe_expert_fwd": (ctypes.c_int, [PP] + [_P] * 7 + [_P]),
             "vmoe_expert_bwd_workspace_size": (ctypes.c_size_t, [PP]),
             "vmoe_expert_bwd": (ctypes.c_int, [PP] + [_P] * 11 + [ctypes.c_size_t, _P]),
+            "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
             "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
             "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
@@ -168,6 +169,17 @@ def vmoe_expert_bwd(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2, workspace, wo
                                      _ptr(w2), _ptr(dye), _ptr(load), _ptr(dxe), _ptr(dw1),
                                      _ptr(dw2), _ptr(workspace), int(workspace_bytes),
                                      _stream(stream)), "vmoe_expert_bwd")
+
+
+VMOE_STATIC_SCRATCH_BYTES = 64 << 20
+
+
+def vmoe_expert_bwd_static_scratch(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2, stream=None):
+    """vmoe_expert_bwd with its dH scratch in the library's own 64 MiB device
+    array, for callers that cannot allocate device memory (see include/vmoe.h)."""
+    _check(library().vmoe_expert_bwd_static_scratch(
+        ctypes.byref(p), _ptr(xe), _ptr(h), _ptr(a), _ptr(w1), _ptr(w2), _ptr(dye), _ptr(load),
+        _ptr(dxe), _ptr(dw1), _ptr(dw2), _stream(stream)), "vmoe_expert_bwd_static_scratch")
 
 
 def vmoe_combine(p, src, weight, expert_idx, slot, dst, stream=None):
