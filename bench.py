@@ -104,6 +104,28 @@ def traffic_record(kernel):
         return None
 
 
+# ----------------------------------------------------------------------------- multi-rank host logic
+def max_over_ranks(values, dist=None, device="cpu"):
+    """Element-wise max of a list of floats over all ranks of the default process
+    group (identity without one).  The job is as slow as its slowest rank."""
+    import torch
+    t = torch.tensor([float(v) for v in values], dtype=torch.float64, device=device)
+    if dist is not None and dist.is_available() and dist.is_initialized():
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return [float(v) for v in t.tolist()]
+
+
+def job_tokens_per_s(tokens_per_rank_step, world, ms_per_step):
+    """Whole-job throughput under weak scaling: every rank runs its own full
+    workload, so the job moves world x tokens_per_rank_step tokens per step."""
+    return tokens_per_rank_step * world / (ms_per_step / 1e3)
+
+
+def rank_weight_seed(rank):
+    """Each rank draws its own experts (independent tasks per rank)."""
+    return 1234 + rank
+
+
 # ----------------------------------------------------------------------------- clocks
 class ClockSampler:
     """nvidia-smi clock / throttle sampling while the timed region runs."""
@@ -176,7 +198,7 @@ def run_ours(args, cfg, rank, world, local_rank):
     # are drawn on the device with the same distribution (rank-dependent seed).
     inp = workloads.make_inputs(cfg, with_weights=False)
     inp = {k2: (None if v is None else v.to(dev)) for k2, v in inp.items()}
-    inp["w1"], inp["w2"] = workloads.make_weights_fast(cfg, dev, seed=1234 + rank)
+    inp["w1"], inp["w2"] = workloads.make_weights_fast(cfg, dev, seed=rank_weight_seed(rank))
     runner = vm.StepRunner(p, inp)
     stream = torch.cuda.current_stream(dev)
 
@@ -246,13 +268,10 @@ def run_ours(args, cfg, rank, world, local_rank):
         raise RuntimeError("device status after timing: " + vm.status_string(st))
 
     # ---- max over ranks
-    times = torch.tensor([ms_total, e2e_s], dtype=torch.float64, device=dev)
-    if dist is not None:
-        dist.all_reduce(times, op=dist.ReduceOp.MAX)
-    ms_total, e2e_s = float(times[0]), float(times[1])
+    ms_total, e2e_s = max_over_ranks([ms_total, e2e_s], dist, dev)
     tokens_per_step = cfg.T * cfg.N * world
     ms_step = ms_total / args.steps
-    value = tokens_per_step / (ms_step / 1e3)
+    value = job_tokens_per_s(cfg.T * cfg.N, world, ms_step)
 
     counts = model_counts(cfg, loads)
     peaks = load_peaks()

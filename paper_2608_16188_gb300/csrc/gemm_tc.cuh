@@ -15,7 +15,9 @@
 //               columns), the fused elementwise step (GELU, or GELU' of an H
 //               prefetched into registers one chunk ahead), bf16 packing, a
 //               per-warp staging tile in shared memory and coalesced 16-byte
-//               row stores.  The accumulator is double buffered in TMEM
+//               row stores (weight gradients, whose tiles are always full:
+//               TMA bulk tensor stores from 128-byte-swizzled staging).
+//               The accumulator is double buffered in TMEM
 //               (2 x BN columns), so tile i's epilogue overlaps tile i+1's
 //               main loop.
 // Tiles are distributed statically: CTA b takes tiles b, b + grid, ...  In
@@ -42,21 +44,25 @@ constexpr int BM = 128;  // rows of one MMA tile (TMEM lanes)
 constexpr int BK = 64;   // K per pipeline slot = one 128-byte swizzle row of bf16
 constexpr int THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
 constexpr int EPI_WARP_BYTES = 32 * 80;  // 32 rows x (64 data + 16 pad) bytes
+constexpr int EPI_WARP_BYTES_TMA = 2 * 4096;  // two 32 x 64 bf16 tiles, 128-byte swizzle
 constexpr int MAX_G = 1024;
 constexpr unsigned long long TIMEOUT_NS = 4000000000ull;
 
 enum { MODE_ROW = 0, MODE_WGRAD = 1 };
 enum { EPI_STORE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
 
-template <int BN>
+template <int BN, int MODE>
 struct Shape {
-    static constexpr int STAGES = BN == 256 ? 4 : 6;
+    // Weight-gradient tiles have K = load <= 2 slots, so 3 slots suffice and
+    // leave room for the double-buffered 128-byte-swizzled TMA-store staging.
+    static constexpr int STAGES = MODE == 1 ? (BN == 256 ? 3 : 4) : (BN == 256 ? 4 : 6);
+    static constexpr int EPI_BYTES = MODE == 1 ? 8 * EPI_WARP_BYTES_TMA : 8 * EPI_WARP_BYTES;
     static constexpr uint32_t A_BYTES = BM * BK * 2;
     static constexpr uint32_t B_BYTES = BN * BK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr uint32_t TMEM_COLS = 2 * BN;
     static constexpr int NUM_BARS = 2 * STAGES + 5;
-    static constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * STAGE_BYTES + 8 * EPI_WARP_BYTES +
+    static constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * STAGE_BYTES + EPI_BYTES +
                                          NUM_BARS * 8 + 16 + THREADS * 4 + (MAX_G + 1) * 4;
 };
 
@@ -140,6 +146,19 @@ __device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2)
         : "memory");
 }
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t src, int c0, int c1,
+                                             int c2) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%2, %3, %4}], [%1];" ::"l"(
+            reinterpret_cast<uint64_t>(map)),
+        "r"(src), "r"(c0), "r"(c1), "r"(c2)
+        : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read1() {
+    asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+}
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
 __device__ __forceinline__ void prefetch_map(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -260,8 +279,8 @@ __device__ __forceinline__ Tile decode_tile(const Args &a, const int *prefix, in
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                    Args args) {
-    using S = Shape<BN>;
+                    const __grid_constant__ CUtensorMap tmD, Args args) {
+    using S = Shape<BN, MODE>;
     constexpr int STAGES = S::STAGES;
     constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
 
@@ -270,7 +289,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
     const uint32_t tiles_addr = smem_u32(smem);
     uint8_t *epi_base = smem + STAGES * S::STAGE_BYTES;
-    uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + 8 * EPI_WARP_BYTES);
+    uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + S::EPI_BYTES);
     int *misc = reinterpret_cast<int *>(bars + S::NUM_BARS);  // [0] tmem base, [1] abort, [2] total
     int *scan_tmp = misc + 4;
     int *prefix = scan_tmp + THREADS;
@@ -487,6 +506,65 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             }
         }
         __syncwarp();
+    } else if (MODE == MODE_WGRAD) {
+        // ------------------------------------------------------------ epilogue (weight gradients)
+        // Warps 2..9 as below, but every tile is full, so each warp writes its
+        // 32 rows x 64 columns into a 128-byte-swizzled staging tile and one
+        // lane stores it with a TMA bulk tensor store (double-buffered).
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int half = ew >> 2;
+        constexpr int COLS = BN / 2;
+        uint8_t *stg = epi_base + ew * EPI_WARP_BYTES_TMA;
+        int nstore = 0;
+        int it = 0;
+        for (int u = blockIdx.x; u < total; u += gridDim.x, ++it) {
+            const Tile t = decode_tile<MODE>(args, prefix, u);
+            const int acc = it & 1;
+            const uint32_t aph = (uint32_t)((it >> 1) & 1);
+            if (!wait_phase(bar_tfull(acc), aph, abort_flag, args.status)) break;
+            tc_fence_after();
+            const int row0 = t.m_blk * BM + q * 32;
+            const int colw = t.n_blk * BN + half * COLS;
+            const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
+                                  (uint32_t)(acc * BN + half * COLS);
+            for (int c = 0; c < COLS; c += 64) {
+                float v[64];
+                if (t.kblocks > 0) {
+                    uint32_t r0[32], r1[32];
+                    tmem_ld32(trow + c, r0);
+                    tmem_ld32(trow + c + 32, r1);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) {
+                        v[i] = __uint_as_float(r0[i]);
+                        v[32 + i] = __uint_as_float(r1[i]);
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) v[i] = 0.0f;
+                }
+                uint8_t *buf = stg + (nstore & 1) * 4096;
+                if (lane == 0 && nstore >= 2) bulk_wait_read1();  // the store that used buf has read it
+                __syncwarp();
+#pragma unroll
+                for (int j = 0; j < 8; ++j)
+                    *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                        f32_to_bf16x8(v + j * 8);
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) {
+                    tma_store_3d(&tmD, smem_u32(buf), colw + c, row0, t.g);
+                    bulk_commit();
+                }
+                ++nstore;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_tempty(acc));
+        }
+        if (lane == 0) bulk_wait_all();
+        __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue
         // Warps 2..9.  Warps w and w+4 share TMEM lane quarter q = w & 3 (rows
@@ -615,9 +693,9 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, 
               uint32_t box_mid);
 
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
-int launch(const CUtensorMap &ma, const CUtensorMap &mb, const Args &a, long long max_tiles,
-           cudaStream_t s, const char *name) {
-    using S = Shape<BN>;
+int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md, const Args &a,
+           long long max_tiles, cudaStream_t s, const char *name) {
+    using S = Shape<BN, MODE>;
     auto kern = grouped_gemm_kernel<BN, MODE, A_MN, B_MN, EPI>;
     static uint64_t attr_done = 0;  // one bit per device
     int dev = 0;
@@ -631,7 +709,7 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const Args &a, long lon
     if (max_tiles <= 0) return VMOE_OK;
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
-    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, a);
+    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, md, a);
     trace_after(s);
     return launch_result();
 }
@@ -670,8 +748,9 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
     a.sD = (long long)C * N;
     a.ldd = N;
     long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
-    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, a, max_tiles, s, name)
-                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, a, max_tiles, s, name);
+    CUtensorMap md = {};  // row mode stores with masked st.global; no output map
+    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, a, max_tiles, s, name)
+                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, a, max_tiles, s, name);
 }
 
 // Weight-gradient GEMM: D[g][M][N] = act1[g][C][M]^T * act2[g][C][N], summed
@@ -682,9 +761,10 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
-    CUtensorMap ma, mb;
+    CUtensorMap ma, mb, md;
     if (!make_map(&ma, act1, M, C, G, 64)) return VMOE_ERR_CUDA;
     if (!make_map(&mb, act2, N, C, G, 64)) return VMOE_ERR_CUDA;
+    if (!make_map(&md, D, N, M, G, 32)) return VMOE_ERR_CUDA;  // 64 x 32 store boxes
     Args a = base_args(p, load);
     a.N = N;
     a.M_fixed = M;
@@ -694,8 +774,8 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     a.sD = (long long)M * N;
     a.ldd = N;
     long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
-    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, a, max_tiles, s, name)
-                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, a, max_tiles, s, name);
+    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, a, max_tiles, s, name)
+                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, a, max_tiles, s, name);
 }
 
 }  // namespace tc

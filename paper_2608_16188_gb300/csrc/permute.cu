@@ -57,16 +57,30 @@ dispatch_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ wei
         int e = idx[row];
         const uint4 *in = reinterpret_cast<const uint4 *>(src + tn * p.d);
         uint4 *out = reinterpret_cast<uint4 *>(dst + (((long long)t * p.E + e) * p.C + s) * p.d);
-        if (weight == nullptr) {
-            for (int v = lane; v < nvec; v += 32) out[v] = __ldg(in + v);
-        } else {
-            float w = weight[row];
-            for (int v = lane; v < nvec; v += 32) {
-                float f[V];
-                Vec<T>::load(__ldg(in + v), f);
+        const float w = weight == nullptr ? 1.0f : weight[row];
+        // All of a lane's loads are issued before its stores (up to UNR 16-byte
+        // vectors per pass) so a warp keeps several row segments in flight.
+        constexpr int UNR = 4;
+        for (int v0 = lane; v0 < nvec; v0 += 32 * UNR) {
+            uint4 buf[UNR];
 #pragma unroll
-                for (int q = 0; q < V; ++q) f[q] *= w;
-                out[v] = Vec<T>::store(f);
+            for (int u = 0; u < UNR; ++u) {
+                int v = v0 + 32 * u;
+                if (v < nvec) buf[u] = __ldg(in + v);
+            }
+#pragma unroll
+            for (int u = 0; u < UNR; ++u) {
+                int v = v0 + 32 * u;
+                if (v >= nvec) continue;
+                if (weight == nullptr) {
+                    out[v] = buf[u];
+                } else {
+                    float f[V];
+                    Vec<T>::load(buf[u], f);
+#pragma unroll
+                    for (int q = 0; q < V; ++q) f[q] *= w;
+                    out[v] = Vec<T>::store(f);
+                }
             }
         }
         return;
@@ -80,7 +94,8 @@ dispatch_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ wei
     for (int v = lane; v < nvec; v += 32) out[v] = make_uint4(0u, 0u, 0u, 0u);
 }
 
-template <typename T>
+// KMAX >= p.k is a compile-time bound so the gathered rows stay in registers.
+template <typename T, int KMAX>
 __global__ void __launch_bounds__(PM_THREADS)
 combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
                const int32_t *__restrict__ idx, const int32_t *__restrict__ slot,
@@ -91,28 +106,52 @@ combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weig
     const int lane = threadIdx.x & 31;
     const int nvec = p.d / V;
     const int t = (int)(tn / p.N);
-    int ej[8], sj[8];
-    float wj[8];
-    for (int j = 0; j < p.k; ++j) {
-        ej[j] = idx[tn * p.k + j];
-        sj[j] = slot[tn * p.k + j];
-        wj[j] = weight ? weight[tn * p.k + j] : 1.0f;
+    float wj[KMAX];
+    const uint4 *rows[KMAX];
+#pragma unroll
+    for (int j = 0; j < KMAX; ++j) {
+        rows[j] = nullptr;
+        wj[j] = 0.0f;
+        if (j < p.k) {
+            const int e = idx[tn * p.k + j], s = slot[tn * p.k + j];
+            wj[j] = weight ? weight[tn * p.k + j] : 1.0f;
+            if (s >= 0)
+                rows[j] = reinterpret_cast<const uint4 *>(
+                    src + (((long long)t * p.E + e) * p.C + s) * p.d);
+        }
     }
     uint4 *out = reinterpret_cast<uint4 *>(dst + tn * p.d);
-    for (int v = lane; v < nvec; v += 32) {
-        float acc[V];
+    // Up to UNR vectors per lane per pass, all k source rows loaded before the
+    // sums, so each warp has k * UNR 16-byte loads in flight.
+    constexpr int UNR = 3;
+    for (int v0 = lane; v0 < nvec; v0 += 32 * UNR) {
+        uint4 buf[KMAX][UNR];
 #pragma unroll
-        for (int q = 0; q < V; ++q) acc[q] = 0.0f;
-        for (int j = 0; j < p.k; ++j) {
-            if (sj[j] < 0) continue;
-            const uint4 *in = reinterpret_cast<const uint4 *>(
-                src + (((long long)t * p.E + ej[j]) * p.C + sj[j]) * p.d);
-            float f[V];
-            Vec<T>::load(__ldg(in + v), f);
+        for (int j = 0; j < KMAX; ++j) {
+            if (rows[j] == nullptr) continue;
 #pragma unroll
-            for (int q = 0; q < V; ++q) acc[q] = fmaf(wj[j], f[q], acc[q]);
+            for (int u = 0; u < UNR; ++u) {
+                int v = v0 + 32 * u;
+                if (v < nvec) buf[j][u] = __ldg(rows[j] + v);
+            }
         }
-        out[v] = Vec<T>::store(acc);
+#pragma unroll
+        for (int u = 0; u < UNR; ++u) {
+            int v = v0 + 32 * u;
+            if (v >= nvec) continue;
+            float acc[V];
+#pragma unroll
+            for (int q = 0; q < V; ++q) acc[q] = 0.0f;
+#pragma unroll
+            for (int j = 0; j < KMAX; ++j) {  // fixed order j = 0..k-1
+                if (rows[j] == nullptr) continue;
+                float f[V];
+                Vec<T>::load(buf[j][u], f);
+#pragma unroll
+                for (int q = 0; q < V; ++q) acc[q] = fmaf(wj[j], f[q], acc[q]);
+            }
+            out[v] = Vec<T>::store(acc);
+        }
     }
 }
 
@@ -134,17 +173,31 @@ int launch_dispatch(const Dims &p, const void *src, const float *weight, const i
     return launch_result();
 }
 
+template <typename T>
+static void combine_as(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+                       const int32_t *slot, void *dst, long long blocks, cudaStream_t s) {
+    const T *in = (const T *)src;
+    T *out = (T *)dst;
+    const unsigned nb = (unsigned)blocks;
+    if (p.k == 1)
+        combine_kernel<T, 1><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+    else if (p.k == 2)
+        combine_kernel<T, 2><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+    else if (p.k <= 4)
+        combine_kernel<T, 4><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+    else
+        combine_kernel<T, 8><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+}
+
 int launch_combine(const Dims &p, const void *src, const float *weight, const int32_t *idx,
                    const int32_t *slot, void *dst, cudaStream_t s) {
     long long rows = (long long)p.T * p.N;
     long long blocks = (rows + PM_WARPS - 1) / PM_WARPS;
     trace_before(s, "combine");
     if (p.bf16)
-        combine_kernel<__nv_bfloat16><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
-            p, (const __nv_bfloat16 *)src, weight, idx, slot, (__nv_bfloat16 *)dst);
+        combine_as<__nv_bfloat16>(p, src, weight, idx, slot, dst, blocks, s);
     else
-        combine_kernel<float><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
-            p, (const float *)src, weight, idx, slot, (float *)dst);
+        combine_as<float>(p, src, weight, idx, slot, dst, blocks, s);
     trace_after(s);
     return launch_result();
 }

@@ -2,7 +2,10 @@
 // capacity scan (Section 2.1 routing, Challenge #1 capacity limits,
 // Section 3.3.1 sequential assignment).
 //
-// Kernel 1 (route_topk): one CTA per (task, tile of TOK tokens).  The logits
+// Kernel 1 (route_topk), bf16 tokens: route_mma_kernel below -- the router
+// product on the tensor cores (mma.sync) with the fp32 weights split into
+// three bf16 parts.  fp32 tokens or given logits: one CTA per (task, tile of
+// TOK tokens) on the CUDA cores.  The logits
 // tile [TOK x E] = x_tile [TOK x d] * W_r[t] [d x E] is accumulated in fp32
 // registers (4 tokens x 4 experts per thread, d swept in chunks of 32 staged
 // in shared memory, one FMA chain per output in increasing i), then written to
@@ -26,7 +29,91 @@ namespace {
 constexpr int RT_THREADS = 256;
 constexpr int RT_KC = 32;  // d-chunk staged per iteration
 
-// ECH experts per pass, TOK tokens per CTA, TOK * ECH = 16 * RT_THREADS.
+// Softmax + top-k of `ntok` logit rows held in shared memory (row pitch ldl),
+// one warp per row: max, softmax denominator, then k rounds of a warp arg-max
+// (larger logit wins, equal logits go to the lower expert index; NaN is
+// treated as -inf so the chosen indices stay in range).
+__device__ __forceinline__ void topk_rows(const Dims &p, const float *lg, int ldl, int ntok, int t,
+                                          int n0, int32_t *__restrict__ out_idx,
+                                          float *__restrict__ out_gate, int nwarps) {
+    const int E = p.E, N = p.N;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool renorm = !(p.flags & VMOE_NO_RENORM);
+    for (int r = warp; r < ntok; r += nwarps) {
+        float v[8];
+        bool taken[8];
+        float mx = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            int e = lane + 32 * i;
+            float val = -INFINITY;
+            if (e < E) {
+                val = lg[r * ldl + e];
+                if (isnan(val)) val = -INFINITY;
+            }
+            v[i] = val;
+            taken[i] = false;
+            mx = fmaxf(mx, val);
+        }
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+        float sum = 0.0f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i)
+            if (lane + 32 * i < E) sum += expf(v[i] - mx);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+
+        float ev[8];
+        int ei[8];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+            ev[j] = 0.0f;
+            ei[j] = 0;
+            if (j >= p.k) continue;
+            float bv = -INFINITY;
+            int be = 0x7fffffff;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                int e = lane + 32 * i;
+                if (e < E && !taken[i] && (v[i] > bv || (v[i] == bv && e < be))) {
+                    bv = v[i];
+                    be = e;
+                }
+            }
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) {
+                float ov = __shfl_xor_sync(0xffffffffu, bv, o);
+                int oe = __shfl_xor_sync(0xffffffffu, be, o);
+                if (ov > bv || (ov == bv && oe < be)) {
+                    bv = ov;
+                    be = oe;
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < 8; ++i)
+                if (lane + 32 * i == be) taken[i] = true;
+            ei[j] = be;
+            ev[j] = expf(bv - mx);
+        }
+        if (lane == 0) {
+            float kept = 0.0f;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < p.k) kept += ev[j];
+            long long base = ((long long)t * N + n0 + r) * p.k;
+#pragma unroll
+            for (int j = 0; j < 8; ++j)
+                if (j < p.k) {
+                    out_idx[base + j] = ei[j];
+                    out_gate[base + j] = renorm ? ev[j] / kept : ev[j] / sum;
+                }
+        }
+    }
+}
+
+// SIMT router for fp32 tokens (or given logits): ECH experts per pass, TOK
+// tokens per CTA, TOK * ECH = 16 * RT_THREADS.
 template <typename TX, int ECH>
 __global__ void __launch_bounds__(RT_THREADS)
 route_topk_kernel(Dims p, const TX *__restrict__ x, const float *__restrict__ wr,
@@ -128,102 +215,213 @@ route_topk_kernel(Dims p, const TX *__restrict__ x, const float *__restrict__ wr
     }
     __syncthreads();
 
-    // Softmax + top-k, one warp per token.
-    const int warp = tid >> 5, lane = tid & 31;
-    const bool renorm = !(p.flags & VMOE_NO_RENORM);
-    for (int r = warp; r < ntok; r += RT_THREADS / 32) {
-        float v[8];
-        bool taken[8];
-        float mx = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            int e = lane + 32 * i;
-            float val = -INFINITY;
-            if (e < E) {
-                val = lg[r * ldl + e];
-                if (isnan(val)) val = -INFINITY;  // NaN never wins a comparison
-            }
-            v[i] = val;
-            taken[i] = false;
-            mx = fmaxf(mx, val);
-        }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-        float sum = 0.0f;
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-            if (lane + 32 * i < E) sum += expf(v[i] - mx);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    topk_rows(p, lg, E + 1, ntok, t, n0, out_idx, out_gate, RT_THREADS / 32);
+}
 
-        float ev[8];
-        int ei[8];
-        for (int j = 0; j < p.k; ++j) {
-            float bv = -INFINITY;
-            int be = 0x7fffffff;
+// Tensor-core router for bf16 tokens.  x is exactly representable in bf16, so
+// x * W_r is formed as x * W_hi + x * W_mid + x * W_lo with the fp32 router
+// weights split into three bf16 parts (W_hi = bf16(W), W_mid = bf16(W - W_hi),
+// W_lo = bf16(W - W_hi - W_mid), together about 24 significant bits): every
+// partial product is exact in fp32 and the mma.sync m16n8k16 instructions
+// accumulate in fp32, so the logits keep fp32 accuracy at a small fraction of
+// the CUDA-core instruction count.  One CTA = 4 warps x 16 tokens of one task;
+// d is swept in chunks of 64 staged in shared memory; the weight split is done
+// while staging, as packed bf16 pairs along k.
+constexpr int RM_TOK = 64;
+constexpr int RM_THREADS = 128;
+constexpr int RM_KC = 64;
+constexpr int RM_XP = RM_KC + 8;  // x row pitch in bf16 (conflict-free fragment loads)
+
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                               uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+__device__ __forceinline__ void split3(float w, __nv_bfloat16 &hi, __nv_bfloat16 &mid,
+                                       __nv_bfloat16 &lo) {
+    hi = __float2bfloat16_rn(w);
+    float r = w - __bfloat162float(hi);
+    mid = __float2bfloat16_rn(r);
+    lo = __float2bfloat16_rn(r - __bfloat162float(mid));
+}
+
+__device__ __forceinline__ uint32_t pack2(__nv_bfloat16 lo_k, __nv_bfloat16 hi_k) {
+    return (uint32_t)__bfloat16_as_ushort(lo_k) | ((uint32_t)__bfloat16_as_ushort(hi_k) << 16);
+}
+
+// NB blocks of 8 experts per pass.
+template <int NB>
+__global__ void __launch_bounds__(RM_THREADS)
+route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__restrict__ wr,
+                 const float *__restrict__ bias, float *__restrict__ logits,
+                 int32_t *__restrict__ out_idx, float *__restrict__ out_gate) {
+    constexpr int NP = NB * 8;
+    constexpr int WP = NP + 8;  // packed-pair row pitch in 32-bit words
+    extern __shared__ __align__(16) uint8_t rm_smem[];
+    __nv_bfloat16 *xs = reinterpret_cast<__nv_bfloat16 *>(rm_smem);            // [64][RM_XP]
+    uint32_t *wp = reinterpret_cast<uint32_t *>(xs + RM_TOK * RM_XP);           // [3][RM_KC/2][WP]
+    float *lg = reinterpret_cast<float *>(wp + 3 * (RM_KC / 2) * WP);           // [64][E+1]
+    const int t = blockIdx.y, n0 = blockIdx.x * RM_TOK;
+    const int E = p.E, d = p.d, N = p.N;
+    const int ldl = E + 1;
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int g = lane >> 2, tq = lane & 3;
+    const int ntok = min(RM_TOK, N - n0);
+    const __nv_bfloat16 *xt = x + ((long long)t * N + n0) * d;
+    const float *wt = wr + (long long)t * d * E;
+    // Per thread and chunk: XV x vectors (16 B each) and WV weight pairs.  The
+    // next chunk's values are loaded into registers before the current chunk's
+    // MMAs run, so global latency overlaps the tensor-core work.
+    constexpr int XV = RM_TOK * (RM_KC / 8) / RM_THREADS;
+    constexpr int WV = (RM_KC / 2) * NP / RM_THREADS;
+    uint4 xv[XV];
+    float wv[WV][2];
+    auto load_chunk = [&](int e0, int k0) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                int e = lane + 32 * i;
-                if (e < E && !taken[i] && (v[i] > bv || (v[i] == bv && e < be))) {
-                    bv = v[i];
-                    be = e;
+        for (int q = 0; q < XV; ++q) {
+            const int i = tid + q * RM_THREADS;
+            const int r = i / (RM_KC / 8), c = (i % (RM_KC / 8)) * 8;
+            xv[q] = make_uint4(0, 0, 0, 0);
+            if (r < ntok && k0 + c < d)
+                xv[q] = __ldg(reinterpret_cast<const uint4 *>(xt + (long long)r * d + k0 + c));
+        }
+#pragma unroll
+        for (int q = 0; q < WV; ++q) {
+            const int i = tid + q * RM_THREADS;
+            const int kp = i / NP, n = i % NP, e = e0 + n, dd = k0 + 2 * kp;
+            wv[q][0] = (e < E && dd < d) ? __ldg(wt + (long long)dd * E + e) : 0.0f;
+            wv[q][1] = (e < E && dd + 1 < d) ? __ldg(wt + (long long)(dd + 1) * E + e) : 0.0f;
+        }
+    };
+    auto stage_chunk = [&]() {
+#pragma unroll
+        for (int q = 0; q < XV; ++q) {
+            const int i = tid + q * RM_THREADS;
+            const int r = i / (RM_KC / 8), c = (i % (RM_KC / 8)) * 8;
+            *reinterpret_cast<uint4 *>(xs + r * RM_XP + c) = xv[q];
+        }
+#pragma unroll
+        for (int q = 0; q < WV; ++q) {
+            const int i = tid + q * RM_THREADS;
+            const int kp = i / NP, n = i % NP;
+            __nv_bfloat16 h0, m0, l0, h1, m1, l1;
+            split3(wv[q][0], h0, m0, l0);
+            split3(wv[q][1], h1, m1, l1);
+            wp[(0 * (RM_KC / 2) + kp) * WP + n] = pack2(h0, h1);
+            wp[(1 * (RM_KC / 2) + kp) * WP + n] = pack2(m0, m1);
+            wp[(2 * (RM_KC / 2) + kp) * WP + n] = pack2(l0, l1);
+        }
+    };
+    for (int e0 = 0; e0 < E; e0 += NP) {
+        float acc[NB][4];
+#pragma unroll
+        for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) acc[nb][i] = 0.0f;
+        load_chunk(e0, 0);
+        for (int k0 = 0; k0 < d; k0 += RM_KC) {
+            __syncthreads();  // the previous chunk's fragments have been read
+            stage_chunk();
+            __syncthreads();
+            if (k0 + RM_KC < d) load_chunk(e0, k0 + RM_KC);
+#pragma unroll
+            for (int ks = 0; ks < RM_KC; ks += 16) {
+                const __nv_bfloat16 *xr = xs + (warp * 16 + g) * RM_XP + ks + 2 * tq;
+                const uint32_t a0 = *reinterpret_cast<const uint32_t *>(xr);
+                const uint32_t a1 = *reinterpret_cast<const uint32_t *>(xr + 8 * RM_XP);
+                const uint32_t a2 = *reinterpret_cast<const uint32_t *>(xr + 8);
+                const uint32_t a3 = *reinterpret_cast<const uint32_t *>(xr + 8 * RM_XP + 8);
+#pragma unroll
+                for (int nb = 0; nb < NB; ++nb) {
+#pragma unroll
+                    for (int sp = 2; sp >= 0; --sp) {  // smallest part first
+                        const uint32_t *wrow = wp + (sp * (RM_KC / 2) + ks / 2 + tq) * WP + nb * 8 + g;
+                        mma_bf16_16816(acc[nb], a0, a1, a2, a3, wrow[0], wrow[4 * WP]);
+                    }
                 }
             }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                int oe = __shfl_xor_sync(0xffffffffu, be, o);
-                if (ov > bv || (ov == bv && oe < be)) {
-                    bv = ov;
-                    be = oe;
-                }
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (lane + 32 * i == be) taken[i] = true;
-            ei[j] = be;
-            ev[j] = expf(bv - mx);
         }
-        if (lane == 0) {
-            float kept = 0.0f;
-            for (int j = 0; j < p.k; ++j) kept += ev[j];
-            long long base = ((long long)t * N + n0 + r) * p.k;
-            for (int j = 0; j < p.k; ++j) {
-                out_idx[base + j] = ei[j];
-                out_gate[base + j] = renorm ? ev[j] / kept : ev[j] / sum;
+#pragma unroll
+        for (int nb = 0; nb < NB; ++nb)
+#pragma unroll
+            for (int i = 0; i < 4; ++i) {
+                const int r = warp * 16 + g + (i >> 1) * 8;
+                const int e = e0 + nb * 8 + 2 * tq + (i & 1);
+                if (r < ntok && e < E) lg[r * ldl + e] = acc[nb][i] + (bias ? bias[(long long)t * E + e] : 0.0f);
             }
-        }
     }
+    __syncthreads();
+    for (int i = tid; i < ntok * E; i += RM_THREADS) {
+        const int r = i / E, e = i - r * E;
+        logits[((long long)t * N + n0 + r) * E + e] = lg[r * ldl + e];
+    }
+    topk_rows(p, lg, ldl, ntok, t, n0, out_idx, out_gate, RM_THREADS / 32);
+}
+
+template <int NB>
+int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, const float *bias,
+                      float *logits, int32_t *idx, float *gate, cudaStream_t s) {
+    constexpr int NP = NB * 8;
+    size_t smem = (size_t)RM_TOK * RM_XP * 2 + (size_t)3 * (RM_KC / 2) * (NP + 8) * 4 +
+                  (size_t)RM_TOK * (p.E + 1) * 4;
+    static uint64_t attr_done = 0;
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 64 && !(attr_done >> dev & 1ull)) {
+        if (cudaFuncSetAttribute(route_mma_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 128 * 1024) != cudaSuccess)
+            return VMOE_ERR_CUDA;
+        attr_done |= 1ull << dev;
+    }
+    dim3 grid((p.N + RM_TOK - 1) / RM_TOK, p.T);
+    trace_before(s, "route_topk");
+    route_mma_kernel<NB><<<grid, RM_THREADS, smem, s>>>(p, x, wr, bias, logits, idx, gate);
+    trace_after(s);
+    return launch_result();
 }
 
 constexpr int CS_THREADS = 256;
 constexpr int CS_WARPS = CS_THREADS / 32;
 
+// SMEM_IDX: the task's idx array and the temporary ranks live in shared memory
+// (read and written with coalesced accesses); otherwise they stay in global memory.
+template <bool SMEM_IDX>
 __global__ void __launch_bounds__(CS_THREADS)
 capacity_scan_kernel(Dims p, const int32_t *__restrict__ idx, int32_t *__restrict__ slot,
                      int32_t *__restrict__ load) {
-    extern __shared__ int cnt[];  // [CS_WARPS][E]
+    extern __shared__ int cs_smem[];
+    int *cnt = cs_smem;  // [CS_WARPS][E]
     const int t = blockIdx.x;
     const int E = p.E, N = p.N, k = p.k, C = p.C;
     const int total = k * N;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long tb = (long long)t * N * k;
+    int *sidx = cs_smem + CS_WARPS * E;  // [N*k] in token-major (memory) order
+    int *srank = sidx + total;           // [N*k]
     for (int i = threadIdx.x; i < CS_WARPS * E; i += CS_THREADS) cnt[i] = 0;
+    if (SMEM_IDX)
+        for (int i = threadIdx.x; i < total; i += CS_THREADS) sidx[i] = idx[tb + i];
     __syncthreads();
+    const int32_t *src = SMEM_IDX ? sidx : idx + tb;
+    int32_t *rank = SMEM_IDX ? srank : slot + tb;
 
     const int per = ((total + CS_WARPS - 1) / CS_WARPS + 31) & ~31;
     const int beg = min(total, warp * per), end = min(total, beg + per);
     int *my = cnt + warp * E;
     const unsigned lt = (1u << lane) - 1u;
-    const long long tb = (long long)t * N * k;
-    // Pass 1: rank within the warp's chunk.
+    // Pass 1: rank within the warp's chunk of the choice-major sequence p = j*N + n.
     for (int p0 = beg; p0 < end; p0 += 32) {
         int pos = p0 + lane;
         bool valid = pos < end;
         int n = valid ? pos % N : 0, j = valid ? pos / N : 0;
-        int e = valid ? idx[tb + (long long)n * k + j] : -1;
+        int e = valid ? src[n * k + j] : -1;
         unsigned peers = __match_any_sync(0xffffffffu, e);
         int before = __popc(peers & lt);
-        if (valid) slot[tb + (long long)n * k + j] = my[e] + before;
+        if (valid) rank[n * k + j] = my[e] + before;
         __syncwarp();
         if (valid && before == 0) my[e] += __popc(peers);
         __syncwarp();
@@ -241,14 +439,25 @@ capacity_scan_kernel(Dims p, const int32_t *__restrict__ idx, int32_t *__restric
     }
     __syncthreads();
     // Pass 2: global rank -> slot.
-    for (int p0 = beg; p0 < end; p0 += 32) {
-        int pos = p0 + lane;
-        if (pos < end) {
-            int n = pos % N, j = pos / N;
-            long long a = tb + (long long)n * k + j;
-            int e = idx[a];
-            int r = slot[a] + my[e];
-            slot[a] = r < C ? r : -1;
+    if (SMEM_IDX) {
+        // each memory position i = n*k + j belongs to the warp whose chunk holds p = j*N + n
+        for (int i = threadIdx.x; i < total; i += CS_THREADS) {
+            const int n = i / k, j = i - n * k;
+            const int pos = j * N + n;
+            const int w = pos / per;
+            const int r = srank[i] + cnt[w * E + sidx[i]];
+            slot[tb + i] = r < C ? r : -1;
+        }
+    } else {
+        for (int p0 = beg; p0 < end; p0 += 32) {
+            int pos = p0 + lane;
+            if (pos < end) {
+                int n = pos % N, j = pos / N;
+                long long a = tb + (long long)n * k + j;
+                int e = idx[a];
+                int r = slot[a] + my[e];
+                slot[a] = r < C ? r : -1;
+            }
         }
     }
 }
@@ -278,19 +487,35 @@ int launch_route(const Dims &p, const void *x, const float *w_router, const floa
                  float *logits, int32_t *idx, float *gate, int32_t *slot, int32_t *load,
                  cudaStream_t s) {
     int st;
-    if (p.bf16) {
+    if (p.bf16 && x != nullptr) {
         const __nv_bfloat16 *xb = (const __nv_bfloat16 *)x;
-        st = p.E <= 32 ? launch_topk<__nv_bfloat16, 32>(p, xb, w_router, bias, logits, idx, gate, s)
-                       : launch_topk<__nv_bfloat16, 64>(p, xb, w_router, bias, logits, idx, gate, s);
+        st = p.E <= 32 ? launch_mma_router<4>(p, xb, w_router, bias, logits, idx, gate, s)
+                       : launch_mma_router<8>(p, xb, w_router, bias, logits, idx, gate, s);
+    } else if (p.bf16) {  // given logits: no GEMV
+        st = launch_topk<__nv_bfloat16, 64>(p, nullptr, w_router, bias, logits, idx, gate, s);
     } else {
         const float *xf = (const float *)x;
         st = p.E <= 32 ? launch_topk<float, 32>(p, xf, w_router, bias, logits, idx, gate, s)
                        : launch_topk<float, 64>(p, xf, w_router, bias, logits, idx, gate, s);
     }
     if (st != VMOE_OK) return st;
-    size_t smem = sizeof(int) * (size_t)CS_WARPS * p.E;
+    const size_t total = (size_t)p.N * p.k;
+    const size_t smem_small = sizeof(int) * (size_t)CS_WARPS * p.E;
+    const size_t smem_big = smem_small + sizeof(int) * 2 * total;
     trace_before(s, "capacity_scan");
-    capacity_scan_kernel<<<p.T, CS_THREADS, smem, s>>>(p, idx, slot, load);
+    if (smem_big <= 96 * 1024) {
+        static uint64_t attr_done = 0;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev < 64 && !(attr_done >> dev & 1ull)) {
+            cudaFuncSetAttribute(capacity_scan_kernel<true>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+            attr_done |= 1ull << dev;
+        }
+        capacity_scan_kernel<true><<<p.T, CS_THREADS, smem_big, s>>>(p, idx, slot, load);
+    } else {
+        capacity_scan_kernel<false><<<p.T, CS_THREADS, smem_small, s>>>(p, idx, slot, load);
+    }
     trace_after(s);
     return launch_result();
 }
