@@ -9,9 +9,9 @@
 // tile [TOK x E] = x_tile [TOK x d] * W_r[t] [d x E] is accumulated in fp32
 // registers (4 tokens x 4 experts per thread, d swept in chunks of 32 staged
 // in shared memory, one FMA chain per output in increasing i), then written to
-// shared memory and to `logits`.  One warp per token then takes the max, the
-// softmax denominator and k rounds of a warp arg-max (larger logit wins, ties
-// to the lower expert index).
+// shared memory and to `logits`.  One thread per token then takes the max,
+// the softmax denominator and the k largest logits (ties to the lower expert
+// index).
 //
 // Kernel 2 (capacity_scan): one CTA per task.  The choice-major assignment
 // sequence p = j*N + n is cut into one contiguous chunk per warp; each warp
@@ -29,86 +29,62 @@ namespace {
 constexpr int RT_THREADS = 256;
 constexpr int RT_KC = 32;  // d-chunk staged per iteration
 
-// Softmax + top-k of `ntok` logit rows held in shared memory (row pitch ldl),
-// one warp per row: max, softmax denominator, then k rounds of a warp arg-max
-// (larger logit wins, equal logits go to the lower expert index; NaN is
-// treated as -inf so the chosen indices stay in range).
+// Softmax + top-k of `ntok` logit rows held in shared memory (row pitch ldl,
+// odd, so the per-thread rows hit distinct banks), one thread per row: the max,
+// the softmax denominator, then k picks, each the best expert that comes after
+// the previous pick in the order (larger logit first, equal logits by lower
+// index).  NaN is treated as -inf so the chosen indices stay in range.
 __device__ __forceinline__ void topk_rows(const Dims &p, const float *lg, int ldl, int ntok, int t,
                                           int n0, int32_t *__restrict__ out_idx,
-                                          float *__restrict__ out_gate, int nwarps) {
+                                          float *__restrict__ out_gate, int nthreads) {
     const int E = p.E, N = p.N;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const bool renorm = !(p.flags & VMOE_NO_RENORM);
-    for (int r = warp; r < ntok; r += nwarps) {
-        float v[8];
-        bool taken[8];
+    for (int r = threadIdx.x; r < ntok; r += nthreads) {
+        const float *row = lg + r * ldl;
         float mx = -INFINITY;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            int e = lane + 32 * i;
-            float val = -INFINITY;
-            if (e < E) {
-                val = lg[r * ldl + e];
-                if (isnan(val)) val = -INFINITY;
-            }
-            v[i] = val;
-            taken[i] = false;
-            mx = fmaxf(mx, val);
+        for (int e = 0; e < E; ++e) {
+            float v = row[e];
+            mx = fmaxf(mx, isnan(v) ? -INFINITY : v);
         }
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
         float sum = 0.0f;
-#pragma unroll
-        for (int i = 0; i < 8; ++i)
-            if (lane + 32 * i < E) sum += expf(v[i] - mx);
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
-
+        for (int e = 0; e < E; ++e) {
+            float v = row[e];
+            sum += expf((isnan(v) ? -INFINITY : v) - mx);
+        }
         float ev[8];
         int ei[8];
+        float pv = INFINITY;  // previous pick: (pv, pe); the next pick comes after it
+        int pe = -1;
+        float kept = 0.0f;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
             ev[j] = 0.0f;
             ei[j] = 0;
             if (j >= p.k) continue;
             float bv = -INFINITY;
-            int be = 0x7fffffff;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-                int e = lane + 32 * i;
-                if (e < E && !taken[i] && (v[i] > bv || (v[i] == bv && e < be))) {
-                    bv = v[i];
+            int be = -1;
+            for (int e = 0; e < E; ++e) {
+                float v = row[e];
+                v = isnan(v) ? -INFINITY : v;
+                const bool after = v < pv || (v == pv && e > pe);
+                if (after && (be < 0 || v > bv)) {  // strict '>' keeps the lower index on ties
+                    bv = v;
                     be = e;
                 }
             }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-                int oe = __shfl_xor_sync(0xffffffffu, be, o);
-                if (ov > bv || (ov == bv && oe < be)) {
-                    bv = ov;
-                    be = oe;
-                }
-            }
-#pragma unroll
-            for (int i = 0; i < 8; ++i)
-                if (lane + 32 * i == be) taken[i] = true;
             ei[j] = be;
             ev[j] = expf(bv - mx);
+            kept += ev[j];
+            pv = bv;
+            pe = be;
         }
-        if (lane == 0) {
-            float kept = 0.0f;
+        const long long base = ((long long)t * N + n0 + r) * p.k;
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                if (j < p.k) kept += ev[j];
-            long long base = ((long long)t * N + n0 + r) * p.k;
-#pragma unroll
-            for (int j = 0; j < 8; ++j)
-                if (j < p.k) {
-                    out_idx[base + j] = ei[j];
-                    out_gate[base + j] = renorm ? ev[j] / kept : ev[j] / sum;
-                }
-        }
+        for (int j = 0; j < 8; ++j)
+            if (j < p.k) {
+                out_idx[base + j] = ei[j];
+                out_gate[base + j] = renorm ? ev[j] / kept : ev[j] / sum;
+            }
     }
 }
 
@@ -215,7 +191,7 @@ route_topk_kernel(Dims p, const TX *__restrict__ x, const float *__restrict__ wr
     }
     __syncthreads();
 
-    topk_rows(p, lg, E + 1, ntok, t, n0, out_idx, out_gate, RT_THREADS / 32);
+    topk_rows(p, lg, E + 1, ntok, t, n0, out_idx, out_gate, RT_THREADS);
 }
 
 // Tensor-core router for bf16 tokens.  x is exactly representable in bf16, so
@@ -359,7 +335,7 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
         const int r = i / E, e = i - r * E;
         logits[((long long)t * N + n0 + r) * E + e] = lg[r * ldl + e];
     }
-    topk_rows(p, lg, ldl, ntok, t, n0, out_idx, out_gate, RM_THREADS / 32);
+    topk_rows(p, lg, ldl, ntok, t, n0, out_idx, out_gate, RM_THREADS);
 }
 
 template <int NB>
