@@ -141,8 +141,10 @@ int vmoe_dispatch(const vmoe_problem *p, const void *src, const float *weight,
 int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const void *w2,
                     const int32_t *load, void *h, void *a, void *ye, void *cuda_stream);
 
-/* Device bytes of scratch vmoe_expert_bwd needs for `p` (the dH buffer,
- * T*E*C*d_ff elements of p->dtype), or 0 if `p` is invalid.  Host only. */
+/* Device bytes of scratch vmoe_expert_bwd needs for `p`, or 0 if `p` is
+ * invalid.  Host only.  It holds dH: T*E*C*d_ff fp32 elements for fp32
+ * problems; for bf16, 2*T*E*C*d_ff bf16 elements, dH kept as a bf16 value plus
+ * its bf16 residual so the weight gradients of small groups stay accurate. */
 size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p);
 
 /* Expert FFN backward (adaptation of the expert weights, Section 3.1), the
@@ -197,6 +199,15 @@ int vmoe_combine(const vmoe_problem *p, const void *src, const float *weight,
  * vmoe_status (VMOE_ERR_DEVICE_TIMEOUT after a kernel gave up a bounded
  * wait).  Synchronises the current device.  `reset` != 0 clears the word. */
 int vmoe_device_status(int reset);
+
+/* Self-test of the failure path: launches one kernel that waits on a device
+ * barrier nothing ever signals, through the same bounded wait the grouped GEMM
+ * uses, and gives up after `limit_ns` nanoseconds (1 ns .. 1 s).  The wait
+ * running out sets the device status word to VMOE_ERR_DEVICE_TIMEOUT (read and
+ * cleared with vmoe_device_status) and the kernel returns normally, leaving the
+ * context usable.  Returns VMOE_OK after the launch, VMOE_ERR_INVALID for a
+ * limit out of range. */
+int vmoe_selftest_bounded_wait(long long limit_ns, void *cuda_stream);
 
 /* Kernel trace (host-side tracing aid).  While enabled on the calling host
  * thread, every kernel the library launches is bracketed by two CUDA events

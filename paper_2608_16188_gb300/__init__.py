@@ -35,7 +35,8 @@ VMOE_GELU_TANH = 1 << 2
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
            "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine",
-           "vmoe_device_status", "vmoe_trace_enable", "vmoe_trace_disable", "vmoe_trace_get")
+           "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
+           "vmoe_trace_disable", "vmoe_trace_get")
 
 
 class VmoeError(RuntimeError):
@@ -78,6 +79,7 @@ def library():
             "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
             "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
+            "vmoe_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_longlong, _P]),
             "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
             "vmoe_trace_disable": (ctypes.c_int, []),
             "vmoe_trace_get": (ctypes.c_int, [ctypes.c_int, ctypes.POINTER(ctypes.c_char_p),
@@ -189,6 +191,11 @@ def vmoe_combine(p, src, weight, expert_idx, slot, dst, stream=None):
 
 def vmoe_device_status(reset: bool = False) -> int:
     return library().vmoe_device_status(1 if reset else 0)
+
+
+def vmoe_selftest_bounded_wait(limit_ns: int, stream=None):
+    _check(library().vmoe_selftest_bounded_wait(int(limit_ns), _stream(stream)),
+           "vmoe_selftest_bounded_wait")
 
 
 def vmoe_trace_enable(max_records: int):

@@ -200,8 +200,9 @@ int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const
 size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p) {
     Dims d;
     if (check_problem(p, &d) != VMOE_OK) return 0;
-    size_t elem = d.bf16 ? 2 : 4;
-    return (size_t)d.T * d.E * d.C * d.f * elem;
+    // bf16: dH as a (bf16 part, bf16 residual) pair per element; fp32: dH itself.
+    size_t per_elem = d.bf16 ? 2 * 2 : 4;
+    return (size_t)d.T * d.E * d.C * d.f * per_elem;
 }
 
 int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,

@@ -86,11 +86,13 @@ struct Args {
     int tiles_n;  // N / BN
     int tiles_m;  // weight-gradient mode: M_fixed / BM; row mode: ceil(C / BM)
     const int32_t *load;
-    __nv_bfloat16 *D;          // output
-    __nv_bfloat16 *D2;         // EPI_GELU: A = GELU(H)
+    __nv_bfloat16 *D;          // output (EPI_DGELU: the bf16 part of dH)
+    __nv_bfloat16 *D2;         // EPI_GELU: A = GELU(H); EPI_DGELU: the bf16 residual of dH
     const __nv_bfloat16 *aux;  // EPI_DGELU: H
-    long long sD;              // group stride of D / D2 / aux (elements)
+    long long sD;              // group stride of D / D2 (elements)
+    long long sAux;            // group stride of aux (elements)
     int ldd;                   // row stride of D / D2 / aux (elements)
+    int ksplit;                // weight-gradient mode: B holds [hi rows; lo rows] (K doubled)
     int gelu_tanh;
     int *status;
 };
@@ -129,14 +131,15 @@ __device__ __forceinline__ unsigned long long global_ns() {
 }
 // Bounded wait for the phase of parity `parity` of barrier `bar`.
 static __device__ __noinline__ bool wait_phase(uint32_t bar, uint32_t parity, volatile int *abort_flag,
-                                        int *status) {
+                                               int *status,
+                                               unsigned long long limit_ns = TIMEOUT_NS) {
     if (mbar_try_wait(bar, parity)) return true;
     const unsigned long long t0 = global_ns();
     for (uint32_t i = 1;; ++i) {
         if (mbar_try_wait(bar, parity)) return true;
         if ((i & 63u) == 0) {
             if (*abort_flag) return false;
-            if (global_ns() - t0 > TIMEOUT_NS) {
+            if (global_ns() - t0 > limit_ns) {
                 *abort_flag = 1;
                 if (status) atomicExch(status, (int)VMOE_ERR_DEVICE_TIMEOUT);
                 return false;
@@ -174,6 +177,14 @@ __device__ __forceinline__ void bulk_wait_read0() {
     asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map, uint32_t bar,
+                                            int c0, int c1, int c2, int c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
 __device__ __forceinline__ void prefetch_map(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }
@@ -257,6 +268,7 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn, bool 
 
 struct Tile {
     int g, m_blk, n_blk, kblocks, kvalid, rows_valid;
+    int khalf;  // weight-gradient mode: k-blocks per half (kblocks = 2 * khalf with ksplit)
 };
 
 template <int MODE>
@@ -285,7 +297,8 @@ __device__ __forceinline__ Tile decode_tile(const Args &a, const int *prefix, in
         int L = __ldg(a.load + t.g);
         L = L < 0 ? 0 : (L > a.C ? a.C : L);
         t.kvalid = L;
-        t.kblocks = (L + BK - 1) / BK;
+        t.khalf = (L + BK - 1) / BK;
+        t.kblocks = a.ksplit ? 2 * t.khalf : t.khalf;
         t.rows_valid = a.M_fixed;
     }
     return t;
@@ -410,23 +423,24 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const uint32_t sa = tiles_addr + stage * S::STAGE_BYTES;
                     const uint32_t sb = sa + S::A_BYTES;
                     const uint32_t fb = bar_full(stage);
-                    mbar_expect_tx(fb, S::STAGE_BYTES);
                     if (MODE == MODE_ROW) {
+                        mbar_expect_tx(fb, S::STAGE_BYTES);
                         tma_load_3d(sa, &tmA, fb, kb * BK, t.m_blk * BM, t.g);
-                        if (B_MN) {
-#pragma unroll
-                            for (int c = 0; c < BN / 64; ++c)
-                                tma_load_3d(sb + c * 8192, &tmB, fb, t.n_blk * BN + c * 64, kb * BK, t.g);
+                        if (B_MN) {  // one 4-D box: BN/64 column chunks of 64 rows
+                            tma_load_4d(sb, &tmB, fb, 0, kb * BK, t.n_blk * (BN / 64), t.g);
                         } else {
                             tma_load_3d(sb, &tmB, fb, kb * BK, t.n_blk * BN, t.g);
                         }
                     } else {
-#pragma unroll
-                        for (int c = 0; c < BM / 64; ++c)
-                            tma_load_3d(sa + c * 8192, &tmA, fb, t.m_blk * BM + c * 64, kb * BK, t.g);
-#pragma unroll
-                        for (int c = 0; c < BN / 64; ++c)
-                            tma_load_3d(sb + c * 8192, &tmB, fb, t.n_blk * BN + c * 64, kb * BK, t.g);
+                        // Weight gradients: K = the group's rows.  With ksplit the second
+                        // half of the k-blocks pairs the same A rows with B's residual
+                        // rows, which start at row C of the group.
+                        mbar_expect_tx(fb, S::STAGE_BYTES);
+                        const int hi = (kb >= t.khalf) ? 1 : 0;
+                        const int ka = (kb - hi * t.khalf) * BK;
+                        const int kbr = hi * args.C + ka;
+                        tma_load_4d(sa, &tmA, fb, 0, ka, t.m_blk * (BM / 64), t.g);
+                        tma_load_4d(sb, &tmB, fb, 0, kbr, t.n_blk * (BN / 64), t.g);
                     }
                     issued[stage]++;
                     if (++stage == STAGES) {
@@ -474,11 +488,11 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 const uint32_t sa = tiles_addr + stage * S::STAGE_BYTES;
                 const uint32_t sb = sa + S::A_BYTES;
                 int nk = BK / 16;
-                if (MODE == MODE_WGRAD && kb == t.kblocks - 1) {
+                if (MODE == MODE_WGRAD && (kb == t.kblocks - 1 || kb == t.khalf - 1)) {
                     // K tail: the MMA reads rows [0, 16*nk) of the slot; rows
                     // [rem, 16*nk) lie past this group's load and are zeroed in
                     // both operands (one 128-byte line per K row per 64-wide chunk).
-                    const int rem = t.kvalid - kb * BK;
+                    const int rem = t.kvalid - (kb - (kb >= t.khalf ? t.khalf : 0)) * BK;
                     nk = (rem + 15) >> 4;
                     const int z0 = rem, z1 = nk * 16;
                     if (z0 < z1) {
@@ -596,7 +610,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int half = ew >> 2;
         constexpr int COLS = BN / 2;
         constexpr int NSC = COLS / 32;  // 32-column sub-chunks per warp
-        constexpr int NOUT = EPI == EPI_GELU ? 2 : 1;
+        constexpr int NOUT = (EPI == EPI_GELU || EPI == EPI_DGELU) ? 2 : 1;
         uint8_t *stg = epi_base + ew * EPI_WARP_BYTES_TMA;
         const bool tanh_form = args.gelu_tanh != 0;
         const int sub_r = lane >> 3, sub_c = lane & 7;  // read-back mapping: 4 rows x 8 x 16 B
@@ -605,7 +619,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int r0 = tl.m_blk * BM + q * 32;
             if (r0 + lane < tl.rows_valid) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
-                    args.aux + (long long)tl.g * args.sD + (long long)(r0 + lane) * args.ldd +
+                    args.aux + (long long)tl.g * args.sAux + (long long)(r0 + lane) * args.ldd +
                     tl.n_blk * BN + half * COLS + sc * 32);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
@@ -702,12 +716,16 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
 #pragma unroll
                         for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i], tanh_form);
                         write_sw(bufA, (sc & 1) * 4, v);
+                    } else if (EPI == EPI_DGELU) {
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) v[i] -= __bfloat162float(__float2bfloat16_rn(v[i]));
+                        write_sw(bufA, (sc & 1) * 4, v);
                     }
                     if ((sc & 1) == 1) {
                         const int c64 = (sc >> 1) * 64;
                         flush(bufD, &tmD, args.D + gofs + c64, colw + c64, row0, t.g, nvalid);
                         ++nstore;
-                        if (EPI == EPI_GELU) {
+                        if (NOUT == 2) {
                             flush(bufA, &tmD2, args.D2 + gofs + c64, colw + c64, row0, t.g, nvalid);
                             ++nstore;
                         }
@@ -746,7 +764,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int r0 = tl.m_blk * BM + q * 32;
             if (r0 + lane < tl.rows_valid) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
-                    args.aux + (long long)tl.g * args.sD + (long long)(r0 + lane) * args.ldd +
+                    args.aux + (long long)tl.g * args.sAux + (long long)(r0 + lane) * args.ldd +
                     tl.n_blk * BN + half * COLS + c * 32);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
@@ -815,6 +833,19 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     for (int i = 0; i < 4; ++i)
                         *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(v + i * 8);
                     store_rows(args.D + gofs + c * 32, nvalid);
+                    if (EPI == EPI_DGELU) {  // residual v - bf16(v): dH = hi + lo to ~16 bits
+#pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            float lv[8];
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) {
+                                const float x = v[i * 8 + e];
+                                lv[e] = x - __bfloat162float(__float2bfloat16_rn(x));
+                            }
+                            *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(lv);
+                        }
+                        store_rows(args.D2 + gofs + c * 32, nvalid);
+                    }
                     if (EPI == EPI_GELU) {
 #pragma unroll
                         for (int i = 0; i < 4; ++i) {
@@ -850,7 +881,15 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
 // Encodes a rank-3 bf16 tensor map {inner, mid, outer} (inner contiguous) with
 // a {64, box_mid, 1} box and 128-byte swizzle; out-of-range elements read 0.
 bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, uint64_t outer,
-              uint32_t box_mid);
+              uint32_t box_mid, uint64_t outer_stride_elems = 0);
+
+// Encodes a rank-4 view of a [outer][rows][mn] bf16 tensor whose mn axis is cut
+// into 64-element chunks: dims {64, rows, mn/64, outer}.  A {64, box_rows,
+// box_chunks, 1} box then lands in shared memory chunk-major -- box_chunks
+// tiles of box_rows x 128 bytes (128-byte swizzle) -- which is the MN-major
+// operand layout, in one copy instead of one per chunk.
+bool make_map_chunked(CUtensorMap *map, const void *base, uint64_t mn, uint64_t rows,
+                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks);
 
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
 int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
@@ -887,16 +926,19 @@ inline Args base_args(const Dims &p, const int32_t *load) {
 
 // Row-mode GEMM: D[g][C rows][N] = act[g][C][K] * B, B MN-major ([K][N]) or
 // K-major ([N][K]).
+// sD / sAux / sAct: group strides (elements) of D and D2, of aux, and of act;
+// 0 means the dense [G, C, width] layout.
 template <int EPI, bool B_MN>
 int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16 *w, int N,
-                    const int32_t *load, __nv_bfloat16 *D, __nv_bfloat16 *D2,
-                    const __nv_bfloat16 *aux, cudaStream_t s, const char *name) {
+             const int32_t *load, __nv_bfloat16 *D, __nv_bfloat16 *D2, const __nv_bfloat16 *aux,
+             cudaStream_t s, const char *name, long long sD = 0, long long sAux = 0,
+             long long sAct = 0) {
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
     CUtensorMap ma, mb;
-    if (!make_map(&ma, act, K, C, G, 128)) return VMOE_ERR_CUDA;
-    bool okb = B_MN ? make_map(&mb, w, N, K, G, 64) : make_map(&mb, w, K, N, G, BN);
+    if (!make_map(&ma, act, K, C, G, 128, (uint64_t)sAct)) return VMOE_ERR_CUDA;
+    bool okb = B_MN ? make_map_chunked(&mb, w, N, K, G, 64, BN / 64) : make_map(&mb, w, K, N, G, BN);
     if (!okb) return VMOE_ERR_CUDA;
     Args a = base_args(p, load);
     a.N = N;
@@ -906,13 +948,14 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
     a.D = D;
     a.D2 = D2;
     a.aux = aux;
-    a.sD = (long long)C * N;
+    a.sD = sD ? sD : (long long)C * N;
+    a.sAux = sAux ? sAux : (long long)C * N;
     a.ldd = N;
     long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
     CUtensorMap md = {}, md2 = {};  // output maps: 64 x 32 store boxes over [G, C, N]
     if (UseTmaStore<MODE_ROW, EPI>::value) {
-        if (!make_map(&md, D, N, C, G, 32)) return VMOE_ERR_CUDA;
-        if (D2 && !make_map(&md2, D2, N, C, G, 32)) return VMOE_ERR_CUDA;
+        if (!make_map(&md, D, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
+        if (D2 && !make_map(&md2, D2, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
     }
     return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, a, max_tiles, s, name)
                 : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, a, max_tiles, s, name);
@@ -920,15 +963,17 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
 
 // Weight-gradient GEMM: D[g][M][N] = act1[g][C][M]^T * act2[g][C][N], summed
 // over each group's load[g] rows; both operands MN-major.
+// ksplit: act2 is [G, 2C, N] -- a bf16 part in rows [0, C) and its residual in
+// rows [C, 2C) -- and D = act1^T (hi + lo), the K loop running over both halves.
 inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __nv_bfloat16 *act2,
                       int N, const int32_t *load, __nv_bfloat16 *D, cudaStream_t s,
-                      const char *name) {
+                      const char *name, bool ksplit = false) {
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
     CUtensorMap ma, mb, md;
-    if (!make_map(&ma, act1, M, C, G, 64)) return VMOE_ERR_CUDA;
-    if (!make_map(&mb, act2, N, C, G, 64)) return VMOE_ERR_CUDA;
+    if (!make_map_chunked(&ma, act1, M, C, G, 64, BM / 64)) return VMOE_ERR_CUDA;
+    if (!make_map_chunked(&mb, act2, N, ksplit ? 2 * C : C, G, 64, BN / 64)) return VMOE_ERR_CUDA;
     if (!make_map(&md, D, N, M, G, 32)) return VMOE_ERR_CUDA;  // 64 x 32 store boxes
     Args a = base_args(p, load);
     a.N = N;
@@ -938,6 +983,7 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     a.D = D;
     a.sD = (long long)M * N;
     a.ldd = N;
+    a.ksplit = ksplit ? 1 : 0;
     long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
     return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name)
                 : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name);

@@ -26,14 +26,28 @@ static EncodeTiledFn encoder() {
 }
 
 bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, uint64_t outer,
-              uint32_t box_mid) {
+              uint32_t box_mid, uint64_t outer_stride_elems) {
     EncodeTiledFn fn = encoder();
     if (!fn) return false;
     cuuint64_t dims[3] = {inner, mid, outer};
-    cuuint64_t strides[2] = {inner * 2, inner * mid * 2};
+    cuuint64_t strides[2] = {inner * 2, (outer_stride_elems ? outer_stride_elems : inner * mid) * 2};
     cuuint32_t box[3] = {64, box_mid, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void *>(base), dims, strides,
+                    box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+bool make_map_chunked(CUtensorMap *map, const void *base, uint64_t mn, uint64_t rows,
+                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks) {
+    EncodeTiledFn fn = encoder();
+    if (!fn || mn % 64 != 0) return false;
+    cuuint64_t dims[4] = {64, rows, mn / 64, outer};
+    cuuint64_t strides[3] = {mn * 2, 128, rows * mn * 2};  // bytes: row, chunk, group
+    cuuint32_t box[4] = {64, box_rows, box_chunks, 1};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,
                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;

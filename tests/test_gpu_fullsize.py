@@ -1,4 +1,5 @@
-"""Full-size parity: the 17-task ViT-B step and the Zipf-skewed step, in the launch
+"""Full-size parity: the 17-task ViT-B step, the Zipf-skewed step, the 6-task ViT-B
+step (two row tiles per group) and the 4-task ViT-S step (128-wide column tiles), in the launch
 configuration the benchmark times, checked against the fp64 oracle.
 
 Routing is compared bit-exactly for every token of every task.  The expert FFN
@@ -8,7 +9,7 @@ the fullest group and, where present, an empty one.  Dispatch and combine are
 checked on whole tasks, and at full size through the property that they move and
 gate-weight rows only (the oracle's combine of the GPU's own expert outputs).  As in the small cases,
 each stage's oracle gets the inputs the GPU call got, and every (task, expert)
-group or task is its own output for the RMS normalisation.
+group, or token row of y and dX, is its own output for the RMS normalisation.
 """
 import numpy as np
 import pytest
@@ -35,7 +36,7 @@ def _ok(name, g, r, mask=None, errs=None, groups=None):
     return e[0] <= BF16_TOL and e[1] <= BF16_RMS_TOL
 
 
-@pytest.mark.parametrize("name", ["vitb_t17", "skew_t8"])
+@pytest.mark.parametrize("name", ["vitb_t17", "skew_t8", "vitb_t6", "vits_t4"])
 def test_fullsize_sampled_parity(name):
     cfg = workloads.CONFIGS[name]
     inp = workloads.make_inputs(cfg)
@@ -68,9 +69,9 @@ def test_fullsize_sampled_parity(name):
 
     # combine at full size from the GPU's own expert outputs
     y_ref = oracle.combine(b.ye, rgate, ridx, rslot, N)
-    assert _ok("y", b.y, y_ref, errs=errs, groups=T), errs
+    assert _ok("y", b.y, y_ref, errs=errs, groups=T * N), errs
     dx_ref = oracle.combine(b.dxe, None, ridx, rslot, N)
-    assert _ok("dx", b.dx, dx_ref, errs=errs, groups=T), errs
+    assert _ok("dx", b.dx, dx_ref, errs=errs, groups=T * N), errs
 
     # sampled groups through the whole expert FFN, forward and backward
     G = T * E

@@ -4,7 +4,8 @@ Routing indices, slots and loads must match bit-exactly when the oracle routes
 from the GPU's own fp32 logits; gates within 1e-6 relative.  Every other output
 of every ABI call must be within 2e-2 (bf16) or 1e-5 (fp32) of the oracle given
 the same inputs, the error of each element normalised by max(rms, |ref|) of its
-own (task, expert) output; y and dX also end to end against the pure oracle.
+own output -- a (task, expert) group's slice of an expert tensor, or one token's
+row of y and dX; y and dX also end to end against the pure oracle.
 The small cases span several tiles in M, N and K with ragged tails, drops, empty
 groups and both N-tile widths of the tensor-core path.
 """
@@ -75,10 +76,10 @@ def _compare_step(cfg, inp_cpu, b, flags):
     assert np.array_equal(np64(xe_g), ref["xe"])  # dispatch is a pure copy
     checks = {  # name: (gpu, reference, row mask, number of separate outputs)
         "dye": (dye_g, s_dye, None, G), "h": (h_g, s_h, rows, G), "a": (a_g, s_a, rows, G),
-        "ye": (ye_g, s_ye, rows, G), "y_stage": (b.y, s_y, None, T),
+        "ye": (ye_g, s_ye, rows, G), "y_stage": (b.y, s_y, None, T * N),
         "dxe": (dxe_g, s_dxe, rows, G), "dw1": (b.dw1, s_dw1, None, G),
-        "dw2": (b.dw2, s_dw2, None, G), "dx_stage": (b.dx, s_dx, None, T),
-        "y_e2e": (b.y, ref["y"], None, T), "dx_e2e": (b.dx, ref["dx"], None, T),
+        "dw2": (b.dw2, s_dw2, None, G), "dx_stage": (b.dx, s_dx, None, T * N),
+        "y_e2e": (b.y, ref["y"], None, T * N), "dx_e2e": (b.dx, ref["dx"], None, T * N),
     }
     errs = {n: (rel_err(g, r, m, gr), rms_err(g, r, m, gr)) for n, (g, r, m, gr) in checks.items()}
     # end-to-end weight gradients: aggregate bar (their inputs A and dYe are bf16 by the ABI)
