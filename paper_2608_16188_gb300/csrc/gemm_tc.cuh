@@ -55,8 +55,9 @@ enum { EPI_STORE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
 // swizzled staging need 64 KB of shared memory, which leaves room for 3
 // pipeline slots at BN 256 instead of 4.  Measured on GB300 at the 17-task
 // ViT-B step: they pay for the weight gradients (always-full tiles, write-
-// bound) and for FC1 + GELU (two outputs per tile); the read-bound row GEMMs
-// with one output (FC2, dA, dX) are faster with 4 slots and masked st.global.
+// bound) and for FC1 + GELU (two outputs per tile); FC2, dX and dA + GELU'
+// (which also writes two outputs, dH and its residual, but reads H) are
+// faster with 4 slots and masked st.global.
 template <int MODE, int EPI>
 struct UseTmaStore {
     static constexpr bool value = MODE == 1 || EPI == 1;
@@ -184,6 +185,10 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *map
         " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
         "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
         : "memory");
+}
+// Named barrier over `count` threads (ids 1..15; 0 is __syncthreads).
+__device__ __forceinline__ void named_bar(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 __device__ __forceinline__ void prefetch_map(const CUtensorMap *map) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
@@ -538,9 +543,10 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         __syncwarp();
     } else if (MODE == MODE_WGRAD) {
         // ------------------------------------------------------------ epilogue (weight gradients)
-        // Warps 2..9 as below, but every tile is full, so each warp writes its
-        // 32 rows x 64 columns into a 128-byte-swizzled staging tile and one
-        // lane stores it with a TMA bulk tensor store (double-buffered).
+        // Every tile is full.  Each warp reads all BN/2 accumulator columns of its
+        // 32 rows with back-to-back tcgen05.ld before one wait, then writes 64-
+        // column chunks into a 128-byte-swizzled 32 x 64 staging tile that one
+        // lane stores with a TMA bulk tensor store (two tiles alternate).
         const int ew = warp - 2;
         const int q = warp & 3;
         const int half = ew >> 2;
@@ -558,40 +564,43 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int colw = t.n_blk * BN + half * COLS;
             const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
                                   (uint32_t)(acc * BN + half * COLS);
-            for (int c = 0; c < COLS; c += 64) {
-                float v[64];
-                if (t.kblocks > 0) {
-                    uint32_t r0[32], r1[32];
-                    tmem_ld32(trow + c, r0);
-                    tmem_ld32(trow + c + 32, r1);
-                    tmem_ld_wait();
+            uint32_t r[COLS / 32][32];
+            if (t.kblocks > 0) {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) {
-                        v[i] = __uint_as_float(r0[i]);
-                        v[32 + i] = __uint_as_float(r1[i]);
-                    }
-                } else {
+                for (int i = 0; i < COLS / 32; ++i) tmem_ld32(trow + i * 32, r[i]);
+                tmem_ld_wait();
+            } else {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) v[i] = 0.0f;
-                }
+                for (int i = 0; i < COLS / 32; ++i)
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) r[i][j] = 0u;
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar_tempty(acc));  // the accumulator is in registers now
+#pragma unroll
+            for (int c = 0; c < COLS / 64; ++c) {
                 uint8_t *buf = stg + (nstore & 1) * 4096;
                 if (lane == 0 && nstore >= 2) bulk_wait_read1();  // the store that used buf has read it
                 __syncwarp();
 #pragma unroll
-                for (int j = 0; j < 8; ++j)
-                    *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                        f32_to_bf16x8(v + j * 8);
+                for (int j = 0; j < 8; ++j) {
+                    const uint32_t *src = &r[2 * c + (j >> 2)][(j & 3) * 8];
+                    uint4 pk;
+                    pk.x = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
+                    pk.y = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
+                    pk.z = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
+                    pk.w = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+                    *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) = pk;
+                }
                 fence_proxy_async();
                 __syncwarp();
                 if (lane == 0) {
-                    tma_store_3d(&tmD, smem_u32(buf), colw + c, row0, t.g);
+                    tma_store_3d(&tmD, smem_u32(buf), colw + c * 64, row0, t.g);
                     bulk_commit();
                 }
                 ++nstore;
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_tempty(acc));
         }
         if (lane == 0) bulk_wait_all();
         __syncwarp();
@@ -876,6 +885,313 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
 }
 
 // ---------------------------------------------------------------------------
+// Weight gradients with the B operand resident ("B-stationary"), for groups of
+// at most 128 rows (C <= 128).
+//
+//   D[g][m-tile][n-tile] = A[g][K rows][m-tile]^T  B[g][K rows][n-tile]
+//
+// One work unit = (group g, column tile n, a run of up to MCH row tiles m).
+// The unit's B tile -- all K rows, and with KSPLIT the residual rows after
+// them -- is loaded once into a resident region and reused by every row tile
+// of the run, whose A tiles stream through a two-deep ring.  Against the
+// streaming kernel this cuts the L2 -> SM traffic of a 128 x 256 output tile
+// from (A + B) per tile to A per tile plus B / MCH.  Roles, TMEM double
+// buffering, bounded waits and the TMA-store epilogue are as in
+// grouped_gemm_kernel.
+template <int BN, bool KSPLIT>
+struct BStatShape {
+    static constexpr int MCH = 6;                              // row tiles per unit
+    static constexpr uint32_t A_KB = BM * BK * 2;              // one A k-block (16 KB)
+    static constexpr uint32_t B_KB = BN * BK * 2;              // one B k-block
+    static constexpr uint32_t A_BUF = 2 * A_KB;                // up to 128 K rows
+    static constexpr uint32_t B_BYTES = (KSPLIT ? 4 : 2) * B_KB;
+    static constexpr int STG_BUFS = KSPLIT ? 1 : 2;            // 32 x 64 staging tiles per warp
+    static constexpr uint32_t EPI_BYTES = 8 * STG_BUFS * 4096;
+    static constexpr uint32_t TMEM_COLS = 2 * BN;
+    static constexpr int NUM_BARS = 11;
+    static constexpr size_t SMEM_BYTES =
+        1024 + B_BYTES + 2 * A_BUF + EPI_BYTES + NUM_BARS * 8 + 16;
+};
+
+template <int BN, bool KSPLIT>
+__global__ void __launch_bounds__(THREADS, 1)
+wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                   const __grid_constant__ CUtensorMap tmD, Args args) {
+    using S = BStatShape<BN, KSPLIT>;
+    constexpr uint32_t IDESC = idesc_bf16(BM, BN, true, true);
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw_addr = smem_u32(smem_raw);
+    uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
+    uint8_t *b_res = smem;                                  // [hi kb0, hi kb1, lo kb0, lo kb1]
+    uint8_t *a_ring = b_res + S::B_BYTES;                   // 2 x [kb0, kb1]
+    uint8_t *epi_base = a_ring + 2 * S::A_BUF;
+    uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + S::EPI_BYTES);
+    int *misc = reinterpret_cast<int *>(bars + S::NUM_BARS);  // [0] tmem base, [1] abort
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const uint32_t bar_bfull = smem_u32(bars + 0), bar_bempty = smem_u32(bars + 1);
+    auto bar_afull = [&](int i) { return smem_u32(bars + 2 + i); };
+    auto bar_aempty = [&](int i) { return smem_u32(bars + 4 + i); };
+    auto bar_tfull = [&](int i) { return smem_u32(bars + 6 + i); };
+    auto bar_tempty = [&](int i) { return smem_u32(bars + 8 + i); };
+    const uint32_t bar_drain = smem_u32(bars + 10);
+    volatile int *abort_flag = misc + 1;
+
+    if (tid == 0) {
+        mbar_init(bar_bfull, 1);
+        mbar_init(bar_bempty, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar_afull(i), 1);
+            mbar_init(bar_aempty(i), 1);
+            mbar_init(bar_tfull(i), 1);
+            mbar_init(bar_tempty(i), 8);
+        }
+        mbar_init(bar_drain, 1);
+        misc[1] = 0;
+        fence_barrier_init();
+        fence_proxy_async();
+        prefetch_map(&tmA);
+        prefetch_map(&tmB);
+        prefetch_map(&tmD);
+    }
+    if (warp == 0) {
+        tmem_alloc(smem_u32(misc), S::TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = (uint32_t)misc[0];
+    const int nch = (args.tiles_m + S::MCH - 1) / S::MCH;
+    const int total = args.G * args.tiles_n * nch;
+    // unit u -> group, column tile, first row tile and row-tile count
+    auto decode = [&](int u, int &g, int &n_blk, int &m0, int &mcnt, int &L) {
+        g = u / (args.tiles_n * nch);
+        const int r = u - g * args.tiles_n * nch;
+        n_blk = r / nch;
+        m0 = (r - n_blk * nch) * S::MCH;
+        mcnt = min(S::MCH, args.tiles_m - m0);
+        L = __ldg(args.load + g);
+        L = L < 0 ? 0 : (L > args.C ? args.C : L);
+    };
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ producer
+        if (lane == 0) {
+            uint32_t bph = 0;
+            int ia = 0;
+            bool ok = true;
+            int b_issued = 0, a_issued[2] = {0, 0};
+            for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+                int g, n_blk, m0, mcnt, L;
+                decode(u, g, n_blk, m0, mcnt, L);
+                const int nkb = (L + BK - 1) / BK;
+                if (nkb == 0) continue;
+                if (!wait_phase(bar_bempty, bph ^ 1u, abort_flag, args.status)) break;
+                mbar_expect_tx(bar_bfull, (uint32_t)(nkb * (KSPLIT ? 2 : 1)) * S::B_KB);
+                for (int kb = 0; kb < nkb; ++kb) {
+                    tma_load_4d(smem_u32(b_res) + kb * S::B_KB, &tmB, bar_bfull, 0, kb * BK,
+                                n_blk * (BN / 64), g);
+                    if (KSPLIT)
+                        tma_load_4d(smem_u32(b_res) + (2 + kb) * S::B_KB, &tmB, bar_bfull, 0,
+                                    args.C + kb * BK, n_blk * (BN / 64), g);
+                }
+                ++b_issued;
+                bph ^= 1u;
+                for (int m = m0; m < m0 + mcnt; ++m, ++ia) {
+                    const int ab = ia & 1;
+                    if (!wait_phase(bar_aempty(ab), (uint32_t)((ia >> 1) & 1) ^ 1u, abort_flag,
+                                    args.status)) {
+                        ok = false;
+                        break;
+                    }
+                    mbar_expect_tx(bar_afull(ab), (uint32_t)nkb * S::A_KB);
+                    for (int kb = 0; kb < nkb; ++kb)
+                        tma_load_4d(smem_u32(a_ring) + ab * S::A_BUF + kb * S::A_KB, &tmA,
+                                    bar_afull(ab), 0, kb * BK, m * (BM / 64), g);
+                    ++a_issued[ab];
+                }
+            }
+            if (*abort_flag) {  // let copies in flight land before the CTA exits
+                const unsigned long long t0 = global_ns();
+                if (b_issued > 0)
+                    while (!mbar_try_wait(bar_bfull, (uint32_t)((b_issued - 1) & 1)) &&
+                           global_ns() - t0 < 100000000ull) {
+                    }
+                for (int i = 0; i < 2; ++i)
+                    if (a_issued[i] > 0)
+                        while (!mbar_try_wait(bar_afull(i), (uint32_t)((a_issued[i] - 1) & 1)) &&
+                               global_ns() - t0 < 200000000ull) {
+                        }
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        uint32_t bph = 0;
+        int ia = 0, it = 0;
+        bool ok = true;
+        // rows [z0, z1) of every 64-wide chunk of a k-block tile are zeroed
+        auto zero_rows = [&](uint8_t *tile, int chunks, int z0, int z1) {
+            const int rows = z1 - z0;
+            const int units = chunks * rows * 8;
+            for (int i = lane; i < units; i += 32) {
+                const int c = i / (rows * 8);
+                const int w = i - c * rows * 8;
+                *reinterpret_cast<uint4 *>(tile + c * 8192 + (z0 + (w >> 3)) * 128 + (w & 7) * 16) =
+                    make_uint4(0, 0, 0, 0);
+            }
+        };
+        for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+            int g, n_blk, m0, mcnt, L;
+            decode(u, g, n_blk, m0, mcnt, L);
+            const int nkb = (L + BK - 1) / BK;
+            const int rem = L - (nkb - 1) * BK;       // valid rows of the last k-block
+            const int nk_last = (rem + 15) >> 4;      // MMAs (K = 16) in the last k-block
+            if (nkb > 0) {
+                if (!wait_phase(bar_bfull, bph, abort_flag, args.status)) break;
+                tc_fence_after();
+                if (rem < nk_last * 16) {  // K tail of the resident B: zero once per unit
+                    zero_rows(b_res + (nkb - 1) * S::B_KB, BN / 64, rem, nk_last * 16);
+                    if (KSPLIT) zero_rows(b_res + (1 + nkb) * S::B_KB, BN / 64, rem, nk_last * 16);
+                    fence_proxy_async();
+                }
+                __syncwarp();
+            }
+            for (int m = m0; m < m0 + mcnt; ++m, ++it) {
+                const int acc = it & 1;
+                if (!wait_phase(bar_tempty(acc), (uint32_t)((it >> 1) & 1) ^ 1u, abort_flag,
+                                args.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                if (nkb == 0) {
+                    if (lane == 0) mbar_arrive(bar_tfull(acc));
+                    __syncwarp();
+                    continue;
+                }
+                const int ab = ia & 1;
+                if (!wait_phase(bar_afull(ab), (uint32_t)((ia >> 1) & 1), abort_flag, args.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                uint8_t *abuf = a_ring + ab * S::A_BUF;
+                if (rem < nk_last * 16) {
+                    zero_rows(abuf + (nkb - 1) * S::A_KB, BM / 64, rem, nk_last * 16);
+                    fence_proxy_async();
+                }
+                __syncwarp();
+                if (lane == 0) {
+                    const uint32_t dtmem = tmem_base + (uint32_t)(acc * BN);
+                    const uint32_t a0 = smem_u32(abuf), b0 = smem_u32(b_res);
+                    for (int part = 0; part < (KSPLIT ? 2 : 1); ++part)
+                        for (int kb = 0; kb < nkb; ++kb) {
+                            const int nk = kb == nkb - 1 ? nk_last : BK / 16;
+                            const uint32_t at = a0 + kb * S::A_KB;
+                            const uint32_t bt = b0 + (part * 2 + kb) * S::B_KB;
+                            for (int kk = 0; kk < nk; ++kk)
+                                mma_bf16(dtmem, operand_desc(at, kk, true), operand_desc(bt, kk, true),
+                                         IDESC, (part | kb | kk) != 0 ? 1u : 0u);
+                        }
+                    mma_commit(bar_aempty(ab));
+                    mma_commit(bar_tfull(acc));
+                }
+                __syncwarp();
+                ++ia;
+            }
+            if (!ok) break;
+            if (nkb > 0) {
+                if (lane == 0) mma_commit(bar_bempty);  // B may be replaced once these MMAs finish
+                __syncwarp();
+                bph ^= 1u;
+            }
+        }
+        if (lane == 0) {
+            mma_commit(bar_drain);
+            const unsigned long long t0 = global_ns();
+            while (!mbar_try_wait(bar_drain, 0) && global_ns() - t0 < 1000000000ull) {
+            }
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------------------ epilogue
+        const int ew = warp - 2;
+        const int q = warp & 3;
+        const int half = ew >> 2;
+        constexpr int COLS = BN / 2;
+        uint8_t *stg = epi_base + ew * S::STG_BUFS * 4096;
+        int nstore = 0, it = 0;
+        bool ok = true;
+        for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
+            int g, n_blk, m0, mcnt, L;
+            decode(u, g, n_blk, m0, mcnt, L);
+            for (int m = m0; m < m0 + mcnt; ++m, ++it) {
+                const int acc = it & 1;
+                if (!wait_phase(bar_tfull(acc), (uint32_t)((it >> 1) & 1), abort_flag, args.status)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const int row0 = m * BM + q * 32;
+                const int colw = n_blk * BN + half * COLS;
+                const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
+                                      (uint32_t)(acc * BN + half * COLS);
+                // all of this warp's accumulator columns with one wait, then
+                // 32 x 64 chunks through the staging tile(s) and TMA stores
+                uint32_t r[COLS / 32][32];
+                if (L > 0) {
+#pragma unroll
+                    for (int i = 0; i < COLS / 32; ++i) tmem_ld32(trow + i * 32, r[i]);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int i = 0; i < COLS / 32; ++i)
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) r[i][j] = 0u;
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar_tempty(acc));
+#pragma unroll
+                for (int c = 0; c < COLS / 64; ++c) {
+                    uint8_t *buf = stg + (S::STG_BUFS == 2 ? (nstore & 1) * 4096 : 0);
+                    if (lane == 0 && nstore >= S::STG_BUFS) {
+                        if (S::STG_BUFS == 2) bulk_wait_read1();
+                        else bulk_wait_read0();
+                    }
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const uint32_t *src = &r[2 * c + (j >> 2)][(j & 3) * 8];
+                        uint4 pk;
+                        pk.x = pack_bf16x2(__uint_as_float(src[0]), __uint_as_float(src[1]));
+                        pk.y = pack_bf16x2(__uint_as_float(src[2]), __uint_as_float(src[3]));
+                        pk.z = pack_bf16x2(__uint_as_float(src[4]), __uint_as_float(src[5]));
+                        pk.w = pack_bf16x2(__uint_as_float(src[6]), __uint_as_float(src[7]));
+                        *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) = pk;
+                    }
+                    fence_proxy_async();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_3d(&tmD, smem_u32(buf), colw + c * 64, row0, g);
+                        bulk_commit();
+                    }
+                    ++nstore;
+                }
+            }
+        }
+        if (lane == 0) bulk_wait_all();
+        __syncwarp();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem_base, S::TMEM_COLS);
+}
+
+// ---------------------------------------------------------------------------
 // Host side.
 
 // Encodes a rank-3 bf16 tensor map {inner, mid, outer} (inner contiguous) with
@@ -910,6 +1226,28 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
     kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, md, md2, a);
+    trace_after(s);
+    return launch_result();
+}
+
+template <bool KSPLIT>
+int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md, const Args &a,
+                 long long units, cudaStream_t s, const char *name) {
+    using S = BStatShape<256, KSPLIT>;
+    auto kern = wgrad_bstat_kernel<256, KSPLIT>;
+    static uint64_t attr_done = 0;  // one bit per device
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev < 64 && !(attr_done >> dev & 1ull)) {
+        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)S::SMEM_BYTES) != cudaSuccess)
+            return VMOE_ERR_CUDA;
+        attr_done |= 1ull << dev;
+    }
+    if (units <= 0) return VMOE_OK;
+    long long grid = units < num_sms() ? units : num_sms();
+    trace_before(s, name);
+    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, md, a);
     trace_after(s);
     return launch_result();
 }
@@ -984,6 +1322,12 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     a.sD = (long long)M * N;
     a.ldd = N;
     a.ksplit = ksplit ? 1 : 0;
+    if (ksplit && wide && C <= 2 * BK) {  // every group fits one resident B tile
+        const int nch = (a.tiles_m + BStatShape<256, true>::MCH - 1) / BStatShape<256, true>::MCH;
+        const long long units = (long long)G * a.tiles_n * nch;
+        return ksplit ? launch_bstat<true>(ma, mb, md, a, units, s, name)
+                      : launch_bstat<false>(ma, mb, md, a, units, s, name);
+    }
     long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
     return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name)
                 : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name);
