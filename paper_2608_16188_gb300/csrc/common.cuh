@@ -100,4 +100,38 @@ __device__ __forceinline__ float gelu_deriv_f(float h, bool tanh_form) {
     return 0.5f * (1.0f + erff(h * 0.7071067811865476f)) + h * inv_sqrt_2pi * expf(-0.5f * h * h);
 }
 
+// Fast exact-form GELU for the bf16 epilogues.  erf(x), x >= 0, by the Hastings
+// rational approximation (Abramowitz & Stegun, Handbook of Mathematical
+// Functions, formula 7.1.26): erf(x) = 1 - t (a1 + t (a2 + t (a3 + t (a4 + t a5))))
+// exp(-x^2), t = 1 / (1 + p x), with |error| <= 1.5e-7 -- far below the bf16
+// rounding of the stored outputs.  With x = |h| / sqrt 2 the factor exp(-x^2) =
+// exp(-h^2 / 2) is also the one in the normal density, so GELU' costs one
+// exponential, one reciprocal and a five-term polynomial.
+struct PhiParts {
+    float Phi;  // standard normal CDF at h
+    float E;    // exp(-h^2 / 2)
+};
+__device__ __forceinline__ PhiParts phi_parts(float h) {
+    const float p = 0.3275911f, a1 = 0.254829592f, a2 = -0.284496736f, a3 = 1.421413741f,
+                a4 = -1.453152027f, a5 = 1.061405429f;
+    const float x = fabsf(h) * 0.7071067811865476f;
+    const float t = __fdividef(1.0f, fmaf(p, x, 1.0f));
+    const float poly = t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, a5, a4), a3), a2), a1);
+    const float E = __expf(-0.5f * h * h);
+    const float tail = 0.5f * poly * E;  // = P(Z > |h|)
+    PhiParts r;
+    r.Phi = h >= 0.0f ? 1.0f - tail : tail;
+    r.E = E;
+    return r;
+}
+__device__ __forceinline__ float gelu_fast(float h, bool tanh_form) {
+    if (tanh_form) return gelu_f(h, true);
+    return h * phi_parts(h).Phi;
+}
+__device__ __forceinline__ float gelu_deriv_fast(float h, bool tanh_form) {
+    if (tanh_form) return gelu_deriv_f(h, true);
+    const PhiParts r = phi_parts(h);
+    return fmaf(h * 0.3989422804014327f, r.E, r.Phi);
+}
+
 }  // namespace vmoe

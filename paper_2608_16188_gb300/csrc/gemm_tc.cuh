@@ -717,13 +717,13 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                             float hv[8];
                             bf16x8_to_f32(hcur[i], hv);
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_f(hv[e], tanh_form);
+                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_fast(hv[e], tanh_form);
                         }
                     }
                     write_sw(bufD, (sc & 1) * 4, v);
                     if (EPI == EPI_GELU) {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = gelu_f(v[i], tanh_form);
+                        for (int i = 0; i < 32; ++i) v[i] = gelu_fast(v[i], tanh_form);
                         write_sw(bufA, (sc & 1) * 4, v);
                     } else if (EPI == EPI_DGELU) {
 #pragma unroll
@@ -835,7 +835,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                             float hv[8];
                             bf16x8_to_f32(hcur[i], hv);
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_f(hv[e], tanh_form);
+                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_fast(hv[e], tanh_form);
                         }
                     }
 #pragma unroll
@@ -860,7 +860,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                         for (int i = 0; i < 4; ++i) {
                             float gv[8];
 #pragma unroll
-                            for (int e = 0; e < 8; ++e) gv[e] = gelu_f(v[i * 8 + e], tanh_form);
+                            for (int e = 0; e < 8; ++e) gv[e] = gelu_fast(v[i * 8 + e], tanh_form);
                             *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(gv);
                         }
                         store_rows(args.D2 + gofs + c * 32, nvalid);
