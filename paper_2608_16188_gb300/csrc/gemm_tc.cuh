@@ -905,12 +905,15 @@ struct BStatShape {
     static constexpr uint32_t B_KB = BN * BK * 2;              // one B k-block
     static constexpr uint32_t A_BUF = 2 * A_KB;                // up to 128 K rows
     static constexpr uint32_t B_BYTES = (KSPLIT ? 4 : 2) * B_KB;
+    // A ring depth 2 (measured: a single A buffer, which would leave room for
+    // double-buffered staging with the split, made dW1 26% slower).
+    static constexpr int A_BUFS = 2;
     static constexpr int STG_BUFS = KSPLIT ? 1 : 2;            // 32 x 64 staging tiles per warp
     static constexpr uint32_t EPI_BYTES = 8 * STG_BUFS * 4096;
     static constexpr uint32_t TMEM_COLS = 2 * BN;
     static constexpr int NUM_BARS = 11;
     static constexpr size_t SMEM_BYTES =
-        1024 + B_BYTES + 2 * A_BUF + EPI_BYTES + NUM_BARS * 8 + 16;
+        1024 + B_BYTES + A_BUFS * A_BUF + EPI_BYTES + NUM_BARS * 8 + 16;
 };
 
 template <int BN, bool KSPLIT>
@@ -924,7 +927,7 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     uint8_t *smem = smem_raw + ((1024u - (raw_addr & 1023u)) & 1023u);
     uint8_t *b_res = smem;                                  // [hi kb0, hi kb1, lo kb0, lo kb1]
     uint8_t *a_ring = b_res + S::B_BYTES;                   // 2 x [kb0, kb1]
-    uint8_t *epi_base = a_ring + 2 * S::A_BUF;
+    uint8_t *epi_base = a_ring + S::A_BUFS * S::A_BUF;
     uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + S::EPI_BYTES);
     int *misc = reinterpret_cast<int *>(bars + S::NUM_BARS);  // [0] tmem base, [1] abort
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -998,8 +1001,8 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                 ++b_issued;
                 bph ^= 1u;
                 for (int m = m0; m < m0 + mcnt; ++m, ++ia) {
-                    const int ab = ia & 1;
-                    if (!wait_phase(bar_aempty(ab), (uint32_t)((ia >> 1) & 1) ^ 1u, abort_flag,
+                    const int ab = ia % S::A_BUFS;
+                    if (!wait_phase(bar_aempty(ab), (uint32_t)((ia / S::A_BUFS) & 1) ^ 1u, abort_flag,
                                     args.status)) {
                         ok = false;
                         break;
@@ -1070,8 +1073,8 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     __syncwarp();
                     continue;
                 }
-                const int ab = ia & 1;
-                if (!wait_phase(bar_afull(ab), (uint32_t)((ia >> 1) & 1), abort_flag, args.status)) {
+                const int ab = ia % S::A_BUFS;
+                if (!wait_phase(bar_afull(ab), (uint32_t)((ia / S::A_BUFS) & 1), abort_flag, args.status)) {
                     ok = false;
                     break;
                 }
