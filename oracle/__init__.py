@@ -18,6 +18,8 @@ Parity status (what pins each function, see ``tests/test_oracle_pins.py``):
   dispatch/combine  identity-expert invariant, brute-force scatter on tiny inputs
   expert_fwd/bwd  torch float64 autograd on the dense special case (E=1, k=1,
                   C=N) and central finite differences of the composed forward
+  router_bwd      torch float64 autograd of the whole routed layer (routing fixed,
+                  gates differentiable) and central finite differences
 """
 from __future__ import annotations
 
@@ -65,7 +67,8 @@ def _load():
                                             ctypes.c_double, ctypes.c_int]
             lib.oracle_num_threads.restype = ctypes.c_int
             for name in ("oracle_router_logits", "oracle_route", "oracle_dispatch",
-                         "oracle_expert_fwd", "oracle_combine", "oracle_expert_bwd"):
+                         "oracle_expert_fwd", "oracle_combine", "oracle_expert_bwd",
+                         "oracle_router_bwd"):
                 getattr(lib, name).restype = None
             _lib = lib
     return _lib
@@ -205,6 +208,37 @@ def expert_bwd(xe, h, a, w1, w2, dye, load, flags: int = 0):
                               dw1.ctypes.data_as(_DP), dw2.ctypes.data_as(_DP))
     return (dh.reshape(*lead, C, f), dxe.reshape(*lead, C, d),
             dw1.reshape(*lead, d, f), dw2.reshape(*lead, f, d))
+
+
+def router_bwd(x, w_router, logits, idx, gate, slot, dy, ye, flags: int = 0):
+    """Router backward with routing fixed.  ye [T,E,C,d] (or [G,C,d]).
+
+    Returns (dgate [T,N,k], dlogits [T,N,E], dw_router [T,d,E], dbias [T,E],
+    dx_router [T,N,d]) in float64.
+    """
+    xx, px = _d(_as_np64(x))
+    T, N, d = xx.shape
+    w, pw = _d(_as_np64(w_router))
+    E = w.shape[2]
+    lg, pl = _d(_as_np64(logits))
+    ix, pix = _i(idx)
+    k = ix.shape[2]
+    g, pg = _d(_as_np64(gate))
+    sl, psl = _i(slot)
+    dyy, pdy = _d(_as_np64(dy))
+    y_e = _as_np64(ye)
+    C = y_e.shape[-2]
+    yy, pye = _d(y_e.reshape(T, E, C, d))
+    dgate = np.empty((T, N, k), np.float64)
+    dl = np.empty((T, N, E), np.float64)
+    dw = np.empty((T, d, E), np.float64)
+    db = np.empty((T, E), np.float64)
+    dxr = np.empty((T, N, d), np.float64)
+    _load().oracle_router_bwd(T, N, d, E, k, C, flags, px, pw, pl, pix, pg, psl, pdy, pye,
+                              dgate.ctypes.data_as(_DP), dl.ctypes.data_as(_DP),
+                              dw.ctypes.data_as(_DP), db.ctypes.data_as(_DP),
+                              dxr.ctypes.data_as(_DP))
+    return dgate, dl, dw, db, dxr
 
 
 def step(x, w_router, bias, w1, w2, dy, k: int, C: int, flags: int = 0, logits=None):

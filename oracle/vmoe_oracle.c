@@ -300,3 +300,77 @@ int oracle_num_threads(void)
     return 1;
 #endif
 }
+
+/* Router backward (the adaptation gradient of the gating network: the router
+ * belongs to the visual module that specification-based tuning adapts,
+ * Section 3.1).  Routing -- the chosen experts and the slots -- is piecewise
+ * constant in the logits and is held fixed; the gates are differentiable:
+ *   dgate_j = <dY[t,n], Ye[t, e_j, s_j]> for a kept choice, 0 for a dropped one
+ *             (y does not depend on a dropped choice's gate);
+ *   renormalised gates (the default) are the softmax of the k selected logits,
+ *     dlogit[e_j] = w_j (dgate_j - sum_i w_i dgate_i), 0 for unselected experts;
+ *   V-MoE gates (ORACLE_FLAG_NO_RENORM) are the full softmax p,
+ *     dlogit[e] = p_e (g_e - sum_j w_j dgate_j), g_e = dgate_j if e = e_j else 0;
+ *   logits = x W_r + bias, so dW_r[t] = sum_n x[t,n]^T dlogit[t,n],
+ *     dbias[t] = sum_n dlogit[t,n], dx_router[t,n] = W_r[t] dlogit[t,n]. */
+void oracle_router_bwd(int T, int N, int d, int E, int k, int C, unsigned flags, const double *x,
+                       const double *w_router, const double *logits, const int32_t *idx,
+                       const double *gate, const int32_t *slot, const double *dy, const double *ye,
+                       double *dgate, double *dlogits, double *dw_router, double *dbias,
+                       double *dx_router)
+{
+    long total = (long)T * N;
+#pragma omp parallel for schedule(static)
+    for (long tn = 0; tn < total; ++tn) {
+        int t = (int)(tn / N);
+        const double *dyr = dy + tn * d;
+        double *dl = dlogits + tn * E;
+        double *dg = dgate + tn * k;
+        for (int j = 0; j < k; ++j) {
+            long a = tn * k + j;
+            dg[j] = 0.0;
+            if (slot[a] < 0) continue;
+            const double *row = ye + (((long)t * E + idx[a]) * C + slot[a]) * d;
+            for (int i = 0; i < d; ++i) dg[j] += dyr[i] * row[i];
+        }
+        double s = 0.0;
+        for (int j = 0; j < k; ++j) s += gate[tn * k + j] * dg[j];
+        for (int e = 0; e < E; ++e) dl[e] = 0.0;
+        if (flags & ORACLE_FLAG_NO_RENORM) {
+            const double *l = logits + tn * E;
+            double mx = l[0];
+            for (int e = 1; e < E; ++e)
+                if (l[e] > mx) mx = l[e];
+            double sum = 0.0;
+            for (int e = 0; e < E; ++e) sum += exp(l[e] - mx);
+            for (int e = 0; e < E; ++e) {
+                double g = 0.0;
+                for (int j = 0; j < k; ++j)
+                    if (idx[tn * k + j] == e) g = dg[j];
+                dl[e] = exp(l[e] - mx) / sum * (g - s);
+            }
+        } else {
+            for (int j = 0; j < k; ++j) dl[idx[tn * k + j]] = gate[tn * k + j] * (dg[j] - s);
+        }
+        double *dxr = dx_router + tn * d;
+        const double *wr = w_router + (long)t * d * E;
+        for (int i = 0; i < d; ++i) {
+            double acc = 0.0;
+            for (int e = 0; e < E; ++e) acc += wr[(long)i * E + e] * dl[e];
+            dxr[i] = acc;
+        }
+    }
+#pragma omp parallel for schedule(static)
+    for (int t = 0; t < T; ++t) {
+        double *dw = dw_router + (long)t * d * E;
+        for (long i = 0; i < (long)d * E; ++i) dw[i] = 0.0;
+        for (int e = 0; e < E; ++e) dbias[(long)t * E + e] = 0.0;
+        for (int n = 0; n < N; ++n) {
+            const double *xr = x + ((long)t * N + n) * d;
+            const double *dl = dlogits + ((long)t * N + n) * E;
+            for (int i = 0; i < d; ++i)
+                for (int e = 0; e < E; ++e) dw[(long)i * E + e] += xr[i] * dl[e];
+            for (int e = 0; e < E; ++e) dbias[(long)t * E + e] += dl[e];
+        }
+    }
+}
