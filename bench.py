@@ -80,6 +80,12 @@ def model_counts(cfg, loads):
         "tc_dx": (A * f * el + w + A * d * el, gemm_flops),
         "tc_dw1": (A * (d + f) * el + G * d * f * el, gemm_flops),
         "tc_dw2": (A * (d + f) * el + G * d * f * el, gemm_flops),
+        # router backward (outside the a1..a12 step; timed on its own)
+        "router_grad": (T * N * d * el + A * d * el + 4 * idx_bytes + T * N * E * 4
+                        + (T * N * E * 4 if cfg.flags & 2 else 0), 2.0 * A * d),
+        "router_dw": (T * N * d * el + T * N * E * 4 + T * d * E * 4 + T * E * 4,
+                      2.0 * T * N * d * E),
+        "router_dx": (T * N * E * 4 + T * d * E * 4 + 2 * T * N * d * el, 2.0 * T * N * d * E),
     }
 
 
@@ -263,6 +269,27 @@ def run_ours(args, cfg, rank, world, local_rank):
     if st != 0:
         raise RuntimeError("device status after timing: " + vm.status_string(st))
 
+    # ---- router backward on its own (the gating network's gradient), L2 flushed
+    # between iterations; the trace times each of its kernels
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    rb_steps = max(3, min(args.steps, 100))
+    for _ in range(3):
+        runner.router_backward(stream)
+    vm.vmoe_trace_enable(rb_steps * 3 + 16)
+    for _ in range(rb_steps):
+        flush.zero_()
+        runner.router_backward(stream)
+    torch.cuda.synchronize(dev)
+    rb_rec = vm.vmoe_trace_disable()
+    rb_kernel = {}
+    for i in range(rb_rec):
+        name, ms = vm.vmoe_trace_get(i)
+        rb_kernel.setdefault(name, []).append(ms)
+    del flush
+    st = vm.vmoe_device_status()
+    if st != 0:
+        raise RuntimeError("device status after router backward: " + vm.status_string(st))
+
     # ---- max over ranks
     ms_total, e2e_s = max_over_ranks([ms_total, e2e_s], dist, dev)
     tokens_per_step = cfg.T * cfg.N * world
@@ -294,6 +321,32 @@ def run_ours(args, cfg, rank, world, local_rank):
                 "traffic": traffic_record(dom),
                 "algorithmic_bytes_per_launch": dom_bytes,
                 "peak_source": peaks["source"] + " (MEASURED_PEAKS.json hbm_gbs)"}
+    rb_stats = {}
+    for name, ms_list in rb_kernel.items():
+        avg = sum(ms_list) / len(ms_list)
+        by, fl = counts.get(name, (0, 0.0))
+        rb_stats[name] = {"launches": len(ms_list), "ms_avg": round(avg, 5),
+                          "gb_s": round(by / (avg * 1e-3) / 1e9, 1) if by else None,
+                          "algorithmic_bytes_per_launch": by}
+    rb_ms = sum(v["ms_avg"] for v in rb_stats.values())
+    rb_dom = max(rb_stats, key=lambda n: rb_stats[n]["ms_avg"]) if rb_stats else None
+    router_bwd = None
+    if rb_dom is not None:
+        rb_ach = rb_stats[rb_dom]["gb_s"] or 0.0
+        router_bwd = {
+            "what": "vmoe_router_bwd: dgate, dlogits, dW_r, dbias, dX += dlogits W_r^T "
+                    "(gating-network gradient; not part of the a1..a12 step above)",
+            "ms_per_call": round(rb_ms, 5), "calls": rb_steps,
+            "l2": "flushed (256 MiB write) before every call",
+            "kernels": rb_stats,
+            "roofline": {"kernel": rb_dom, "bound": "hbm", "achieved": rb_ach,
+                         "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                         "frac": round(rb_ach / peaks["hbm_gbs"], 4),
+                         "traffic": traffic_record(rb_dom),
+                         "peak_source": peaks["source"] + " (MEASURED_PEAKS.json hbm_gbs)"},
+            "step_with_router_bwd_tokens_per_s": round(
+                job_tokens_per_s(cfg.T * cfg.N, world, ms_step + rb_ms), 1),
+        }
     gemm_flops = sum(counts[n][1] * kstats[n]["launches_per_step"] for n in kstats if n.startswith("tc_"))
     tflops = gemm_flops / (ms_step * 1e-3) / 1e12 * world
     h2d = (x_h.numel() * x_h.element_size() + dy_h.numel() * dy_h.element_size())
@@ -318,6 +371,7 @@ def run_ours(args, cfg, rank, world, local_rank):
                 "h2d_bytes_per_step": h2d * world, "d2h_bytes_per_step": d2h * world,
                 "steps": e2e_steps},
         "clocks": clocks,
+        "router_bwd": router_bwd,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(cfg, budget_s=args.cpu_budget)

@@ -20,6 +20,7 @@
  *   vmoe_expert_bwd dH = (dYe W2^T) * GELU'(H), dXe = dH W1^T,
  *                  dW1 = Xe^T dH, dW2 = A^T dYe
  *   vmoe_combine   dX  = sum_j dXe[e_j, s_j]
+ *   vmoe_router_bwd dgate, dlogits, dW_r, dbias; dX += dlogits W_r^T
  *
  * Conventions for every entry point:
  *  - Ownership: every array argument is caller-owned DEVICE memory (except
@@ -194,6 +195,33 @@ int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void *xe, const 
  *   dst [T,N,d] out.  The forward uses weight = gate, the backward (dX) NULL. */
 int vmoe_combine(const vmoe_problem *p, const void *src, const float *weight,
                  const int32_t *expert_idx, const int32_t *slot, void *dst, void *cuda_stream);
+
+/* Router backward (Section 3.1 adapts the visual module, its gating network
+ * included; Section 2.1 defines the gates as a softmax of the router logits).
+ * With the routing held fixed (expert_idx, slot from vmoe_route), the gradient
+ * of <dY, y> with y = sum_j gate_j Ye[e_j, s_j]:
+ *   dgate[t,n,j]   = <dY[t,n], Ye[t,e_j,s_j]> for a kept choice, 0 if dropped;
+ *   dlogits[t,n,e] = softmax backward: with s = sum_j gate_j dgate_j,
+ *     renormalised gates:  dlogits[e_j] = gate_j (dgate_j - s), 0 elsewhere;
+ *     VMOE_NO_RENORM:      dlogits[e]   = p_e (dgate(e) - s), p = softmax(logits)
+ *                          and dgate(e) = dgate_j if e = e_j, else 0;
+ *   dw_router[t]   = x[t]^T dlogits[t]      (sum over the N tokens of task t);
+ *   dbias[t,e]     = sum_n dlogits[t,n,e];
+ *   dx[t,n,:]     += W_r[t] dlogits[t,n]    (summed in fp32, rounded once).
+ * Inputs: x, dY [T,N,d] and Ye [T,E,C,d] in p->dtype (Ye is the expert output
+ * of vmoe_expert_fwd); w_router [T,d,E], logits [T,N,E], gate [T,N,k] fp32;
+ * expert_idx, slot [T,N,k] int32.  w_router may be NULL only when dx is NULL;
+ * logits is read only with VMOE_NO_RENORM (else it may be NULL).
+ * Outputs (overwritten): dgate [T,N,k], dlogits [T,N,E], dw_router [T,d,E]
+ * fp32; dbias [T,E] fp32, nullable.  dx [T,N,d] in p->dtype is read and
+ * updated in place (the dX of vmoe_combine, which then holds the input
+ * gradient through both the experts and the router); NULL skips it.
+ * Sums run in fixed orders; no atomics. */
+int vmoe_router_bwd(const vmoe_problem *p, const void *x, const float *w_router,
+                    const float *logits, const int32_t *expert_idx, const float *gate,
+                    const int32_t *slot, const void *dy, const void *ye, float *dgate,
+                    float *dlogits, float *dw_router, float *dbias, void *dx,
+                    void *cuda_stream);
 
 /* Device status word of the current device: 0 when clean, otherwise a
  * vmoe_status (VMOE_ERR_DEVICE_TIMEOUT after a kernel gave up a bounded

@@ -34,7 +34,7 @@ VMOE_GELU_TANH = 1 << 2
 # Every symbol include/vmoe.h declares.
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
-           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine",
+           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd",
            "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
            "vmoe_trace_disable", "vmoe_trace_get")
 
@@ -78,6 +78,7 @@ def library():
             "vmoe_expert_bwd": (ctypes.c_int, [PP] + [_P] * 11 + [ctypes.c_size_t, _P]),
             "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
+            "vmoe_router_bwd": (ctypes.c_int, [PP] + [_P] * 13 + [_P]),
             "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
             "vmoe_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_longlong, _P]),
             "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
@@ -187,6 +188,15 @@ def vmoe_expert_bwd_static_scratch(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2
 def vmoe_combine(p, src, weight, expert_idx, slot, dst, stream=None):
     _check(library().vmoe_combine(ctypes.byref(p), _ptr(src), _ptr(weight), _ptr(expert_idx),
                                   _ptr(slot), _ptr(dst), _stream(stream)), "vmoe_combine")
+
+
+def vmoe_router_bwd(p, x, w_router, logits, expert_idx, gate, slot, dy, ye, dgate, dlogits,
+                    dw_router, dbias=None, dx=None, stream=None):
+    """Router backward with the routing fixed; dx (if given) is updated in place."""
+    _check(library().vmoe_router_bwd(
+        ctypes.byref(p), _ptr(x), _ptr(w_router), _ptr(logits), _ptr(expert_idx), _ptr(gate),
+        _ptr(slot), _ptr(dy), _ptr(ye), _ptr(dgate), _ptr(dlogits), _ptr(dw_router), _ptr(dbias),
+        _ptr(dx), _stream(stream)), "vmoe_router_bwd")
 
 
 def vmoe_device_status(reset: bool = False) -> int:

@@ -179,6 +179,24 @@ int vmoe_combine(const vmoe_problem *p, const void *src, const float *weight,
     return launch_combine(d, src, weight, expert_idx, slot, dst, (cudaStream_t)cuda_stream);
 }
 
+int vmoe_router_bwd(const vmoe_problem *p, const void *x, const float *w_router,
+                    const float *logits, const int32_t *expert_idx, const float *gate,
+                    const int32_t *slot, const void *dy, const void *ye, float *dgate,
+                    float *dlogits, float *dw_router, float *dbias, void *dx,
+                    void *cuda_stream) {
+    Dims d;
+    int st = check_problem(p, &d);
+    if (st != VMOE_OK) return st;
+    if (!dev_ok(x) || !dev_ok(expert_idx) || !dev_ok(gate) || !dev_ok(slot) || !dev_ok(dy) ||
+        !dev_ok(ye) || !dev_ok(dgate) || !dev_ok(dlogits) || !dev_ok(dw_router) ||
+        !opt_ok(dbias) || !opt_ok(dx))
+        return VMOE_ERR_INVALID;
+    if (dx ? !dev_ok(w_router) : !opt_ok(w_router)) return VMOE_ERR_INVALID;
+    if ((p->flags & VMOE_NO_RENORM) ? !dev_ok(logits) : !opt_ok(logits)) return VMOE_ERR_INVALID;
+    return launch_router_bwd(d, x, w_router, logits, expert_idx, gate, slot, dy, ye, dgate,
+                             dlogits, dw_router, dbias, dx, (cudaStream_t)cuda_stream);
+}
+
 int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const void *w2,
                     const int32_t *load, void *h, void *a, void *ye, void *cuda_stream) {
     Dims d;

@@ -51,6 +51,10 @@ int launch_expert_bwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bf
                            const __nv_bfloat16 *w2, const __nv_bfloat16 *dye,
                            const int32_t *load, __nv_bfloat16 *dxe, __nv_bfloat16 *dw1,
                            __nv_bfloat16 *dw2, __nv_bfloat16 *dh, cudaStream_t s);
+int launch_router_bwd(const Dims &p, const void *x, const float *w_router, const float *logits,
+                      const int32_t *idx, const float *gate, const int32_t *slot, const void *dy,
+                      const void *ye, float *dgate, float *dlogits, float *dw_router, float *dbias,
+                      void *dx, cudaStream_t s);
 
 // ---------------------------------------------------------------------------
 // Device helpers.

@@ -2,14 +2,16 @@
 
 Plumbing only: torch allocates the caller-owned device buffers the C ABI writes
 into, and ``StepRunner`` issues the seven library calls of one step in order on
-one stream.  No arithmetic of the method happens here.
+one stream -- eight with the router backward (``router_grad=True``), which adds
+the gradient of the gating network.  No arithmetic of the method happens here.
 """
 from __future__ import annotations
 
 import torch
 
 from . import (VMOE_BF16, vmoe_combine, vmoe_dispatch, vmoe_expert_bwd,
-               vmoe_expert_bwd_workspace_size, vmoe_expert_fwd, vmoe_problem_capacity, vmoe_route)
+               vmoe_expert_bwd_workspace_size, vmoe_expert_fwd, vmoe_problem_capacity, vmoe_route,
+               vmoe_router_bwd)
 
 
 class Buffers:
@@ -38,6 +40,11 @@ class Buffers:
         self.dw1 = e(T, E, d, f)
         self.dw2 = e(T, E, f, d)
         self.dx = e(T, N, d)
+        # router backward
+        self.dgate = e(T, N, k, dtype=f32)
+        self.dlogits = e(T, N, E, dtype=f32)
+        self.dw_router = e(T, d, E, dtype=f32)
+        self.dbias = e(T, E, dtype=f32)
         self.workspace = torch.empty(vmoe_expert_bwd_workspace_size(p), dtype=torch.uint8,
                                      device=device)
 
@@ -46,12 +53,14 @@ class StepRunner:
     """Issues the library calls of one forward + backward step.
 
     ``inputs`` holds device tensors x, dy [T,N,d], w_router [T,d,E], bias [T,E]
-    or None, w1 [T,E,d,f], w2 [T,E,f,d].
+    or None, w1 [T,E,d,f], w2 [T,E,f,d].  With ``router_grad`` the backward also
+    produces dW_r and dbias and adds the router's share to dX.
     """
 
-    def __init__(self, p, inputs, bufs: Buffers | None = None):
+    def __init__(self, p, inputs, bufs: Buffers | None = None, router_grad: bool = False):
         self.p = p
         self.inp = inputs
+        self.router_grad = router_grad
         self.b = bufs if bufs is not None else Buffers(p, inputs["x"].device)
 
     def forward(self, stream=None):
@@ -68,6 +77,13 @@ class StepRunner:
         vmoe_expert_bwd(p, b.xe, b.h, b.a, i["w1"], i["w2"], b.dye, b.load, b.dxe, b.dw1, b.dw2,
                         b.workspace, stream=stream)
         vmoe_combine(p, b.dxe, None, b.idx, b.slot, b.dx, stream)
+        if self.router_grad:
+            self.router_backward(stream)
+
+    def router_backward(self, stream=None):
+        p, i, b = self.p, self.inp, self.b
+        vmoe_router_bwd(p, i["x"], i["w_router"], b.logits, b.idx, b.gate, b.slot, i["dy"], b.ye,
+                        b.dgate, b.dlogits, b.dw_router, b.dbias, b.dx, stream)
 
     def step(self, stream=None):
         self.forward(stream)

@@ -98,6 +98,15 @@ def test_null_and_misaligned_pointers_are_rejected_without_cuda(vm):
     st = lib.vmoe_expert_bwd_static_scratch(ctypes.byref(vm.problem(17, 1576, 768, 3072, 32, 2, 1.25)),
                                             P, P, P, P, P, P, P, P, P, P, None)
     assert st == vm.VMOE_ERR_UNSUPPORTED  # dH larger than the static array
+    # router backward: W_r is required with dx, logits with VMOE_NO_RENORM
+    st = lib.vmoe_router_bwd(ctypes.byref(p), P, None, None, P, P, P, P, P, P, P, P, None, P, None)
+    assert st == vm.VMOE_ERR_INVALID
+    nr = vm.problem(2, 64, 128, 256, 4, 2, 1.25, "bf16", flags=vm.VMOE_NO_RENORM)
+    st = lib.vmoe_router_bwd(ctypes.byref(nr), P, P, None, P, P, P, P, P, P, P, P, None, None, None)
+    assert st == vm.VMOE_ERR_INVALID
+    st = lib.vmoe_router_bwd(ctypes.byref(p), P, None, None, P, P, P, P, P, P, P, P + 8, None, None,
+                             None)
+    assert st == vm.VMOE_ERR_INVALID  # misaligned dW_r
     # bf16: dH as (bf16 value, bf16 residual) pairs
     assert vm.vmoe_expert_bwd_workspace_size(p) == 2 * 4 * oracle.capacity(64, 4, 2, 1.25) * 256 * 2 * 2
     for s in (0, -1, -2, -3, -4, 7):
