@@ -80,12 +80,15 @@ def model_counts(cfg, loads):
         "tc_dx": (A * f * el + w + A * d * el, gemm_flops),
         "tc_dw1": (A * (d + f) * el + G * d * f * el, gemm_flops),
         "tc_dw2": (A * (d + f) * el + G * d * f * el, gemm_flops),
-        # router backward (outside the a1..a12 step; timed on its own)
-        "router_grad": (T * N * d * el + A * d * el + 4 * idx_bytes + T * N * E * 4
-                        + (T * N * E * 4 if cfg.flags & 2 else 0), 2.0 * A * d),
+        # router backward (outside the a1..a12 step; timed on its own).  router_grad:
+        # dY and the kept Ye rows in, dgate and dlogits out, dX read and written,
+        # W_r once per task (logits too without renormalisation).  router_dw: x and
+        # dlogits in, dW_r and dbias out.
+        "router_grad": (3 * T * N * d * el + A * d * el + 4 * idx_bytes + T * N * E * 4
+                        + T * d * E * 4 + (T * N * E * 4 if cfg.flags & 2 else 0),
+                        2.0 * A * d + 2.0 * T * N * k * d),
         "router_dw": (T * N * d * el + T * N * E * 4 + T * d * E * 4 + T * E * 4,
                       2.0 * T * N * d * E),
-        "router_dx": (T * N * E * 4 + T * d * E * 4 + 2 * T * N * d * el, 2.0 * T * N * d * E),
     }
 
 
@@ -270,14 +273,18 @@ def run_ours(args, cfg, rank, world, local_rank):
         raise RuntimeError("device status after timing: " + vm.status_string(st))
 
     # ---- router backward on its own (the gating network's gradient), L2 flushed
-    # between iterations; the trace times each of its kernels
+    # between iterations -- a 256 MiB write, then a 256 MiB read so that the
+    # lines left in L2 are clean and the next call pays no write-back for them;
+    # the trace times each of its kernels
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    flush_r = torch.ones(64 << 20, dtype=torch.float32, device=dev)
     rb_steps = max(3, min(args.steps, 100))
     for _ in range(3):
         runner.router_backward(stream)
     vm.vmoe_trace_enable(rb_steps * 3 + 16)
     for _ in range(rb_steps):
         flush.zero_()
+        flush_r.sum()
         runner.router_backward(stream)
     torch.cuda.synchronize(dev)
     rb_rec = vm.vmoe_trace_disable()
@@ -285,7 +292,7 @@ def run_ours(args, cfg, rank, world, local_rank):
     for i in range(rb_rec):
         name, ms = vm.vmoe_trace_get(i)
         rb_kernel.setdefault(name, []).append(ms)
-    del flush
+    del flush, flush_r
     st = vm.vmoe_device_status()
     if st != 0:
         raise RuntimeError("device status after router backward: " + vm.status_string(st))
@@ -337,7 +344,7 @@ def run_ours(args, cfg, rank, world, local_rank):
             "what": "vmoe_router_bwd: dgate, dlogits, dW_r, dbias, dX += dlogits W_r^T "
                     "(gating-network gradient; not part of the a1..a12 step above)",
             "ms_per_call": round(rb_ms, 5), "calls": rb_steps,
-            "l2": "flushed (256 MiB write) before every call",
+            "l2": "flushed before every call (256 MiB write, then 256 MiB read: clean lines)",
             "kernels": rb_stats,
             "roofline": {"kernel": rb_dom, "bound": "hbm", "achieved": rb_ach,
                          "peak": peaks["hbm_gbs"], "unit": "GB/s",

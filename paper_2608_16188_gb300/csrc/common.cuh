@@ -83,6 +83,30 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
     return *reinterpret_cast<uint32_t *>(&h);
 }
 
+// Warp-level bf16 tensor-core product D += A B, m16n8k16, fp32 accumulate.
+__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
+                                               uint32_t a3, uint32_t b0, uint32_t b1) {
+    asm volatile(
+        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// An fp32 value as three bf16 parts, w ~= hi + mid + lo to about 24 significant
+// bits: each product of a bf16 value with a part is exact in fp32.
+__device__ __forceinline__ void split3(float w, __nv_bfloat16 &hi, __nv_bfloat16 &mid,
+                                       __nv_bfloat16 &lo) {
+    hi = __float2bfloat16_rn(w);
+    float r = w - __bfloat162float(hi);
+    mid = __float2bfloat16_rn(r);
+    lo = __float2bfloat16_rn(r - __bfloat162float(mid));
+}
+
+__device__ __forceinline__ uint32_t pack2(__nv_bfloat16 lo_k, __nv_bfloat16 hi_k) {
+    return (uint32_t)__bfloat16_as_ushort(lo_k) | ((uint32_t)__bfloat16_as_ushort(hi_k) << 16);
+}
+
 // GELU and its derivative: exact erf form by default, tanh form with
 // VMOE_GELU_TANH.  Both call CUDA's erff / expf / tanhf.
 __device__ __forceinline__ float gelu_f(float h, bool tanh_form) {

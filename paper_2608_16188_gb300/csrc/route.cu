@@ -208,27 +208,6 @@ constexpr int RM_THREADS = 128;
 constexpr int RM_KC = 64;
 constexpr int RM_XP = RM_KC + 8;  // x row pitch in bf16 (conflict-free fragment loads)
 
-__device__ __forceinline__ void mma_bf16_16816(float (&c)[4], uint32_t a0, uint32_t a1, uint32_t a2,
-                                               uint32_t a3, uint32_t b0, uint32_t b1) {
-    asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
-        "{%8, %9}, {%0, %1, %2, %3};"
-        : "+f"(c[0]), "+f"(c[1]), "+f"(c[2]), "+f"(c[3])
-        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
-}
-
-__device__ __forceinline__ void split3(float w, __nv_bfloat16 &hi, __nv_bfloat16 &mid,
-                                       __nv_bfloat16 &lo) {
-    hi = __float2bfloat16_rn(w);
-    float r = w - __bfloat162float(hi);
-    mid = __float2bfloat16_rn(r);
-    lo = __float2bfloat16_rn(r - __bfloat162float(mid));
-}
-
-__device__ __forceinline__ uint32_t pack2(__nv_bfloat16 lo_k, __nv_bfloat16 hi_k) {
-    return (uint32_t)__bfloat16_as_ushort(lo_k) | ((uint32_t)__bfloat16_as_ushort(hi_k) << 16);
-}
-
 // NB blocks of 8 experts per pass.
 template <int NB>
 __global__ void __launch_bounds__(RM_THREADS)
