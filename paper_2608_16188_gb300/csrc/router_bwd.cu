@@ -445,7 +445,9 @@ router_grad_fast_kernel(Dims p, const __nv_bfloat16 *__restrict__ dy,
 
 // ---------------------------------------------------------------------------
 // Kernel 2 (bf16): dW_r = x^T dlogit and dbias on the tensor cores.
-constexpr int DW_THREADS = 256;     // 8 warps x 16 rows of d
+constexpr int DW_MT = 2;            // m16 tiles (of d rows) per warp
+constexpr int DW_WARPS = 4;         // DW_WARPS x DW_MT x 16 = DW_BD rows
+constexpr int DW_THREADS = 32 * DW_WARPS;
 constexpr int DW_BD = 128;          // rows of d per CTA
 constexpr int DW_BE = 32;           // experts per CTA
 constexpr int DW_KC = 32;           // tokens per stage
@@ -459,10 +461,11 @@ struct DwSmem {
     __nv_bfloat16 x[DW_STAGES][DW_KC][DW_XP];     // token rows of the d-slice
     float dl[DW_STAGES][DW_KC][DW_BE];            // dlogit rows as loaded (fp32)
     __nv_bfloat16 part[3][DW_BE][DW_PP];          // their three bf16 parts, expert-major
-    float bias[DW_THREADS / 32][DW_BE];
+    float bias[DW_WARPS][DW_BE];
     float bias_sum[DW_BE];
 };
 static_assert(sizeof(DwSmem) <= 48 * 1024, "static shared memory");
+static_assert(DW_WARPS * DW_MT * 16 == DW_BD, "warp tiling of the d-slice");
 static_assert(DW_BD * DW_RP * sizeof(float) <= sizeof(DwSmem::x), "partial tile reuses x");
 
 __device__ __forceinline__ void cp_async16(void *smem, const void *gmem, bool valid) {
@@ -491,7 +494,9 @@ __device__ __forceinline__ void ldsm_x4_t(uint32_t (&r)[4], const void *smem) {
 }
 
 // grid (DW_SPLIT, ceil(d / DW_BD), T * ceil(E / DW_BE)), cluster (DW_SPLIT, 1, 1).
-// Warp w owns rows [16 w, 16 w + 16) of the CTA's d-slice and all 32 experts.
+// Warp w owns rows [32 w, 32 w + 32) of the CTA's d-slice (two m16 tiles, so
+// each dlogit fragment read from shared memory feeds two products) and all 32
+// experts.
 __global__ void __cluster_dims__(DW_SPLIT, 1, 1) __launch_bounds__(DW_THREADS)
 router_dw_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x,
                      const float *__restrict__ dlg, float *__restrict__ dw,
@@ -513,9 +518,9 @@ router_dw_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x,
     const bool do_bias = dbias != nullptr && blockIdx.y == 0;
 
     auto load_x = [&](int chunk, int stage) {
-        // 32 token rows x 16 vectors of 8 bf16: two per thread
+        // 32 token rows x 16 vectors of 8 bf16
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
+        for (int u = 0; u < DW_KC * 16 / DW_THREADS; ++u) {
             const int v = tid + u * DW_THREADS;
             const int r = v >> 4, cv = (v & 15) * 8;
             const int n = n_beg + chunk * DW_KC + r;
@@ -528,29 +533,39 @@ router_dw_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x,
     const bool vec_dl = (E & 3) == 0;
     auto load_dl = [&](int chunk, int stage) {
         if (vec_dl) {
-            const int r = tid >> 3, c4 = (tid & 7) * 4;
-            const int n = n_beg + chunk * DW_KC + r;
-            const bool ok = n < n_end && e0 + c4 < E;
-            cp_async16(&sm.dl[stage][r][c4], ok ? dlt + (long long)n * E + e0 + c4 : dlt, ok);
+#pragma unroll
+            for (int u = 0; u < DW_KC * 8 / DW_THREADS; ++u) {
+                const int v = tid + u * DW_THREADS;
+                const int r = v >> 3, c4 = (v & 7) * 4;
+                const int n = n_beg + chunk * DW_KC + r;
+                const bool ok = n < n_end && e0 + c4 < E;
+                cp_async16(&sm.dl[stage][r][c4], ok ? dlt + (long long)n * E + e0 + c4 : dlt, ok);
+            }
         } else {
 #pragma unroll
-            for (int u = 0; u < 4; ++u) {
-                const int r = (tid >> 5) + 8 * u, c = tid & 31;
+            for (int u = 0; u < DW_KC * DW_BE / DW_THREADS; ++u) {
+                const int v = tid + u * DW_THREADS;
+                const int r = v >> 5, c = v & 31;
                 const int n = n_beg + chunk * DW_KC + r;
                 const bool ok = n < n_end && e0 + c < E;
                 cp_async4(&sm.dl[stage][r][c], ok ? dlt + (long long)n * E + e0 + c : dlt, ok);
             }
         }
     };
-    // the split: this thread's 4 values are expert column tid % 32, token rows tid / 32 + 8u
-    const int pc = tid & 31, pr = tid >> 5;
+    // the split: warp w takes token rows [8 w, 8 w + 8) of the chunk, lane = expert
+    // column, so each part of a lane's 8 tokens is one 16-byte shared store
+    // (rows 80 bytes apart: the 8 lanes of a quarter-warp hit distinct banks)
+    static_assert(DW_KC == 8 * DW_WARPS, "one 8-token row group per warp");
+    const int pc = lane;
     float bias_acc = 0.0f;
 
-    float acc[4][4];
+    float acc[DW_MT][4][4];
 #pragma unroll
-    for (int a = 0; a < 4; ++a)
+    for (int mt = 0; mt < DW_MT; ++mt)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) acc[a][b] = 0.0f;
+        for (int a = 0; a < 4; ++a)
+#pragma unroll
+            for (int b = 0; b < 4; ++b) acc[mt][a][b] = 0.0f;
 
     // prologue: chunks 0 .. STAGES-2
 #pragma unroll
@@ -573,43 +588,64 @@ router_dw_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x,
             }
             cp_async_commit();
         }
+        {
+            uint32_t ph[4], pm[4], pl[4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const float v = sm.dl[stage][pr + 8 * u][pc];
-            __nv_bfloat16 h, m, l;
-            split3(v, h, m, l);
-            sm.part[0][pc][pr + 8 * u] = h;
-            sm.part[1][pc][pr + 8 * u] = m;
-            sm.part[2][pc][pr + 8 * u] = l;
-            bias_acc += v;
+            for (int u = 0; u < 4; ++u) {
+                const float v0 = sm.dl[stage][8 * warp + 2 * u][pc];
+                const float v1 = sm.dl[stage][8 * warp + 2 * u + 1][pc];
+                __nv_bfloat16 h0, m0, l0, h1, m1, l1;
+                split3(v0, h0, m0, l0);
+                split3(v1, h1, m1, l1);
+                ph[u] = pack2(h0, h1);
+                pm[u] = pack2(m0, m1);
+                pl[u] = pack2(l0, l1);
+                bias_acc += v0;
+                bias_acc += v1;
+            }
+            *reinterpret_cast<uint4 *>(&sm.part[0][pc][8 * warp]) = make_uint4(ph[0], ph[1], ph[2], ph[3]);
+            *reinterpret_cast<uint4 *>(&sm.part[1][pc][8 * warp]) = make_uint4(pm[0], pm[1], pm[2], pm[3]);
+            *reinterpret_cast<uint4 *>(&sm.part[2][pc][8 * warp]) = make_uint4(pl[0], pl[1], pl[2], pl[3]);
         }
         __syncthreads();  // parts visible
         // two-level sum: this chunk's products, then into the running total
-        float cacc[4][4];
+        float cacc[DW_MT][4][4];
 #pragma unroll
-        for (int a = 0; a < 4; ++a)
+        for (int mt = 0; mt < DW_MT; ++mt)
 #pragma unroll
-            for (int b = 0; b < 4; ++b) cacc[a][b] = 0.0f;
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b < 4; ++b) cacc[mt][a][b] = 0.0f;
 #pragma unroll
         for (int ks = 0; ks < DW_KC; ks += 16) {
             const int mi = lane >> 3, r = lane & 7;
-            uint32_t a[4];
-            ldsm_x4_t(a, &sm.x[stage][ks + (mi >> 1) * 8 + r][warp * 16 + (mi & 1) * 8]);
+            uint32_t a[DW_MT][4];
+#pragma unroll
+            for (int mt = 0; mt < DW_MT; ++mt)
+                ldsm_x4_t(a[mt], &sm.x[stage][ks + (mi >> 1) * 8 + r]
+                                     [(warp * DW_MT + mt) * 16 + (mi & 1) * 8]);
 #pragma unroll
             for (int part = 0; part < 3; ++part) {
 #pragma unroll
                 for (int np = 0; np < 2; ++np) {
                     uint32_t b[4];
                     ldsm_x4(b, &sm.part[part][np * 16 + (mi >> 1) * 8 + r][ks + (mi & 1) * 8]);
-                    mma_bf16_16816(cacc[2 * np], a[0], a[1], a[2], a[3], b[0], b[1]);
-                    mma_bf16_16816(cacc[2 * np + 1], a[0], a[1], a[2], a[3], b[2], b[3]);
+#pragma unroll
+                    for (int mt = 0; mt < DW_MT; ++mt) {
+                        mma_bf16_16816(cacc[mt][2 * np], a[mt][0], a[mt][1], a[mt][2], a[mt][3],
+                                       b[0], b[1]);
+                        mma_bf16_16816(cacc[mt][2 * np + 1], a[mt][0], a[mt][1], a[mt][2],
+                                       a[mt][3], b[2], b[3]);
+                    }
                 }
             }
         }
 #pragma unroll
-        for (int a = 0; a < 4; ++a)
+        for (int mt = 0; mt < DW_MT; ++mt)
 #pragma unroll
-            for (int b = 0; b < 4; ++b) acc[a][b] += cacc[a][b];
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b < 4; ++b) acc[mt][a][b] += cacc[mt][a][b];
     }
     cp_async_wait<0>();
     __syncthreads();
@@ -619,20 +655,22 @@ router_dw_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x,
     {
         const int g = lane >> 2, q = lane & 3;
 #pragma unroll
-        for (int nt = 0; nt < 4; ++nt) {
-            const int m = warp * 16 + g, n = nt * 8 + 2 * q;
-            red[m * DW_RP + n] = acc[nt][0];
-            red[m * DW_RP + n + 1] = acc[nt][1];
-            red[(m + 8) * DW_RP + n] = acc[nt][2];
-            red[(m + 8) * DW_RP + n + 1] = acc[nt][3];
-        }
+        for (int mt = 0; mt < DW_MT; ++mt)
+#pragma unroll
+            for (int nt = 0; nt < 4; ++nt) {
+                const int m = (warp * DW_MT + mt) * 16 + g, n = nt * 8 + 2 * q;
+                red[m * DW_RP + n] = acc[mt][nt][0];
+                red[m * DW_RP + n + 1] = acc[mt][nt][1];
+                red[(m + 8) * DW_RP + n] = acc[mt][nt][2];
+                red[(m + 8) * DW_RP + n + 1] = acc[mt][nt][3];
+            }
     }
-    if (do_bias) sm.bias[warp][pc] = bias_acc;
+    if (do_bias) sm.bias[warp][pc] = bias_acc;  // warp w's tokens 8w..8w+7 of every chunk
     __syncthreads();
     if (do_bias && tid < DW_BE) {
         float b = 0.0f;
 #pragma unroll
-        for (int w = 0; w < DW_THREADS / 32; ++w) b += sm.bias[w][tid];
+        for (int w = 0; w < DW_WARPS; ++w) b += sm.bias[w][tid];
         sm.bias_sum[tid] = b;
     }
     cluster.sync();
