@@ -85,12 +85,23 @@ constexpr int RG_WARPS = RG_THREADS / 32;
 constexpr int RG_UNROLL = 2;
 constexpr size_t RG_SMEM_CAP = 200 * 1024;
 
-// Shared memory: per-warp dlogit rows (VMOE_NO_RENORM), then W_r[t]^T with a
-// row pitch of d + 4 floats (16-byte aligned rows).
+// Shared memory: per-warp dlogit rows (VMOE_NO_RENORM), then W_r[t]^T, one row
+// per expert with pitch wt_pitch(d) floats.  Within each block of 256 columns the
+// columns are permuted so that the 8 columns 8L..8L+7 a lane reads sit at 4L..4L+3
+// and 128+4L..128+4L+3: the lanes of a warp then read two runs of consecutive
+// 16-byte words, free of bank conflicts.
+__host__ __device__ inline int wt_pitch(int d) { return ((d + 255) & ~255) + 4; }
+__device__ __forceinline__ int wt_col(int i) {  // physical position of column i
+    const int w = i & 255, q = w & 7;
+    return (i & ~255) + ((w >> 3) << 2) + (q < 4 ? q : 124 + q);
+}
+__device__ __forceinline__ int wt_col8(int v) {  // first half of columns v..v+7, v % 8 == 0
+    return (v & ~255) + ((v & 255) >> 1);
+}
 inline size_t rg_smem_rows(const Dims &p) {
     return (p.flags & VMOE_NO_RENORM) ? (size_t)RG_WARPS * p.E * sizeof(float) : 0;
 }
-inline size_t rg_smem_w(const Dims &p) { return (size_t)p.E * (p.d + 4) * sizeof(float); }
+inline size_t rg_smem_w(const Dims &p) { return (size_t)p.E * wt_pitch(p.d) * sizeof(float); }
 
 // W_r[t] ([d][E], fp32) into shared memory as W^T with row pitch dp.  Kept out
 // of line so its load batch does not raise the token loop's register count.
@@ -113,7 +124,7 @@ __device__ __noinline__ void stage_wt(const float *__restrict__ wrt, float *WT, 
 #pragma unroll
                 for (int u = 0; u < RG_UNROLL; ++u)
                     if (e8 + u < E8) {
-                        float *col = WT + (8 * (e8 + u)) * dp + i;
+                        float *col = WT + (8 * (e8 + u)) * dp + wt_col(i);
                         col[0 * dp] = buf[u][0].x;
                         col[1 * dp] = buf[u][0].y;
                         col[2 * dp] = buf[u][0].z;
@@ -127,7 +138,7 @@ __device__ __noinline__ void stage_wt(const float *__restrict__ wrt, float *WT, 
         }
     } else {
         for (int i = threadIdx.x; i < d; i += RG_THREADS)
-            for (int e = 0; e < E; ++e) WT[e * dp + i] = __ldg(wrt + (long long)i * E + e);
+            for (int e = 0; e < E; ++e) WT[e * dp + wt_col(i)] = __ldg(wrt + (long long)i * E + e);
     }
 }
 
@@ -221,8 +232,9 @@ __device__ __forceinline__ void dx_terms(float (&r)[8], int v, int ne, bool nore
         }
         float w[8];
         if (WSMEM) {
-            const float4 *wp = reinterpret_cast<const float4 *>(WT + e * dp + v);
-            const float4 a = wp[0], b = wp[1];
+            const float *wp = WT + e * dp + wt_col8(v);
+            const float4 a = *reinterpret_cast<const float4 *>(wp);
+            const float4 b = *reinterpret_cast<const float4 *>(wp + 128);
             w[0] = a.x; w[1] = a.y; w[2] = a.z; w[3] = a.w;
             w[4] = b.x; w[5] = b.y; w[6] = b.z; w[7] = b.w;
         } else {
@@ -248,7 +260,7 @@ router_grad_kernel(Dims p, const T *__restrict__ dy, const T *__restrict__ ye,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int d = p.d, E = p.E, k = p.k, N = p.N;
     const bool norenorm = (p.flags & VMOE_NO_RENORM) != 0;
-    const int dp = d + 4;
+    const int dp = wt_pitch(d);
     float *dlrow = rg_smem + warp * E;
     float *WT = rg_smem + (norenorm ? RG_WARPS * E : 0);
     const long long TN = (long long)p.T * N;
@@ -330,7 +342,7 @@ router_grad_fast_kernel(Dims p, const __nv_bfloat16 *__restrict__ dy,
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int d = p.d, E = p.E, k = p.k, N = p.N;
     const bool norenorm = (p.flags & VMOE_NO_RENORM) != 0;
-    const int dp = d + 4;
+    const int dp = wt_pitch(d);
     float *dlrow = rg_smem + warp * E;
     float *WT = rg_smem + (norenorm ? RG_WARPS * E : 0);
     const long long TN = (long long)p.T * N;
