@@ -5,8 +5,10 @@
  * V-MoE expert layers (AdaSprite, arxiv 2608.16188):
  *   router logits -> softmax + top-k gating -> per-expert capacity scan ->
  *   dispatch into [T,E,C,d] expert buffers -> expert FFN (Linear-GELU-Linear)
- *   forward -> weighted combine back to token order, and the backward of the
- *   expert path (dX, dW1, dW2) with routing and gates held constant.
+ *   forward -> weighted combine back to token order, the backward of the
+ *   expert path (dX, dW1, dW2) with routing and gates held constant, and the
+ *   router backward (dgate, dlogits, dW_r, dbias and the router's share of dX)
+ *   with the routing held fixed.
  *
  * Only the test suite, the smoke check and the benchmark's CPU-baseline leg
  * may load this file.  It shares no code, header or constant with the CUDA
