@@ -94,16 +94,19 @@ def model_counts(cfg, loads):
 
 def traffic_record(kernel):
     """DRAM bytes per launch of `kernel` from the committed ncu summary
-    (profiles/dram_traffic.json), if the kernel's source file still hashes to the
+    (profiles/dram_traffic.json), if the kernel's source files still hash to the
     value recorded with the counters; else None."""
     import hashlib
     path = os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
         with open(path) as fh:
             rec = json.load(fh)["kernels"][kernel]
-        with open(os.path.join(ROOT, rec["source_file"]), "rb") as fh:
-            if hashlib.sha256(fh.read()).hexdigest() != rec["source_sha256"]:
-                return None
+        h = hashlib.sha256()
+        for f in rec["source_files"]:
+            with open(os.path.join(ROOT, f), "rb") as fh:
+                h.update(fh.read())
+        if h.hexdigest() != rec["sources_sha256"]:
+            return None
         return float(rec["dram_bytes_per_launch_full_size"])
     except Exception:
         return None
