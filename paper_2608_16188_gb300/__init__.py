@@ -224,4 +224,4 @@ def vmoe_trace_get(i: int):
     return name.value.decode(), ms.value
 
 
-from .step import Buffers, StepRunner  # noqa: E402  (needs the names above)
+from .step import Buffers, HostPipeline, StepRunner  # noqa: E402  (needs the names above)

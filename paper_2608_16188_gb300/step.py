@@ -7,6 +7,8 @@ the gradient of the gating network.  No arithmetic of the method happens here.
 """
 from __future__ import annotations
 
+import copy
+
 import torch
 
 from . import (VMOE_BF16, vmoe_combine, vmoe_dispatch, vmoe_expert_bwd,
@@ -88,3 +90,71 @@ class StepRunner:
     def step(self, stream=None):
         self.forward(stream)
         self.backward(stream)
+
+
+class HostPipeline:
+    """Steps from pinned host inputs to pinned host outputs, with the host<->device
+    copies overlapped with compute.
+
+    Two slots each hold device copies of x, dY, y and dX; everything else (weights,
+    activations, gradients) is shared, as the steps run in order on one compute
+    stream.  The copies run on their own stream: step i+1's x and dY upload while
+    step i computes, y of step i is read back while its backward runs, and dX as
+    soon as it is done.  ``weights`` holds w_router, bias, w1, w2 on the device.
+    """
+
+    def __init__(self, p, weights, bufs: Buffers | None = None, device="cuda",
+                 router_grad: bool = False):
+        self.p = p
+        base = bufs if bufs is not None else Buffers(p, device)
+        self.slots = []
+        for _ in range(2):
+            b = copy.copy(base)
+            b.y = torch.empty_like(base.y)
+            b.dx = torch.empty_like(base.dx)
+            inp = dict(weights)
+            inp["x"] = torch.empty_like(base.y)
+            inp["dy"] = torch.empty_like(base.y)
+            self.slots.append(StepRunner(p, inp, b, router_grad=router_grad))
+        self.copy_stream = torch.cuda.Stream(device)
+        ev = lambda: [torch.cuda.Event() for _ in range(2)]  # noqa: E731
+        self.h2d, self.fwd, self.done, self.d2h = ev(), ev(), ev(), ev()
+
+    def _upload(self, slot, x_host, dy_host):
+        r = self.slots[slot]
+        with torch.cuda.stream(self.copy_stream):
+            r.inp["x"].copy_(x_host, non_blocking=True)
+            r.inp["dy"].copy_(dy_host, non_blocking=True)
+        self.h2d[slot].record(self.copy_stream)
+
+    def run(self, inputs, outputs, stream=None):
+        """inputs[i] = (x, dY) and outputs[i] = (y, dX): pinned host tensors of
+        step i.  Enqueues every step and returns; synchronise the copy stream (or
+        the device) before reading the outputs."""
+        cs = stream if stream is not None else torch.cuda.current_stream()
+        steps = len(inputs)
+        if steps == 0:
+            return
+        self._upload(0, *inputs[0])
+        for i in range(steps):
+            s = i % 2
+            r = self.slots[s]
+            cs.wait_event(self.h2d[s])
+            if i >= 2:  # this slot's y / dX of step i-2 have been read back
+                cs.wait_event(self.d2h[s])
+            r.forward(cs)
+            self.fwd[s].record(cs)
+            r.backward(cs)
+            self.done[s].record(cs)
+            if i + 1 < steps:  # the other slot is free once step i-1 has finished
+                if i >= 1:
+                    self.copy_stream.wait_event(self.done[s ^ 1])
+                self._upload(s ^ 1, *inputs[i + 1])
+            y_host, dx_host = outputs[i]
+            self.copy_stream.wait_event(self.fwd[s])
+            with torch.cuda.stream(self.copy_stream):
+                y_host.copy_(r.b.y, non_blocking=True)
+            self.copy_stream.wait_event(self.done[s])
+            with torch.cuda.stream(self.copy_stream):
+                dx_host.copy_(r.b.dx, non_blocking=True)
+            self.d2h[s].record(self.copy_stream)
