@@ -22,6 +22,7 @@
 #include <math.h>
 
 #include "common.cuh"
+#include "topk.cuh"
 
 namespace vmoe {
 namespace {
@@ -30,62 +31,12 @@ constexpr int RT_THREADS = 256;
 constexpr int RT_KC = 32;  // d-chunk staged per iteration
 
 // Softmax + top-k of `ntok` logit rows held in shared memory (row pitch ldl,
-// odd, so the per-thread rows hit distinct banks), one thread per row: the max,
-// the softmax denominator, then k picks, each the best expert that comes after
-// the previous pick in the order (larger logit first, equal logits by lower
-// index).  NaN is treated as -inf so the chosen indices stay in range.
+// odd, so the per-thread rows hit distinct banks), one thread per row.
 __device__ __forceinline__ void topk_rows(const Dims &p, const float *lg, int ldl, int ntok, int t,
                                           int n0, int32_t *__restrict__ out_idx,
                                           float *__restrict__ out_gate, int nthreads) {
-    const int E = p.E, N = p.N;
-    const bool renorm = !(p.flags & VMOE_NO_RENORM);
-    for (int r = threadIdx.x; r < ntok; r += nthreads) {
-        const float *row = lg + r * ldl;
-        float mx = -INFINITY;
-        for (int e = 0; e < E; ++e) {
-            float v = row[e];
-            mx = fmaxf(mx, isnan(v) ? -INFINITY : v);
-        }
-        float sum = 0.0f;
-        for (int e = 0; e < E; ++e) {
-            float v = row[e];
-            sum += expf((isnan(v) ? -INFINITY : v) - mx);
-        }
-        float ev[8];
-        int ei[8];
-        float pv = INFINITY;  // previous pick: (pv, pe); the next pick comes after it
-        int pe = -1;
-        float kept = 0.0f;
-#pragma unroll
-        for (int j = 0; j < 8; ++j) {
-            ev[j] = 0.0f;
-            ei[j] = 0;
-            if (j >= p.k) continue;
-            float bv = -INFINITY;
-            int be = -1;
-            for (int e = 0; e < E; ++e) {
-                float v = row[e];
-                v = isnan(v) ? -INFINITY : v;
-                const bool after = v < pv || (v == pv && e > pe);
-                if (after && (be < 0 || v > bv)) {  // strict '>' keeps the lower index on ties
-                    bv = v;
-                    be = e;
-                }
-            }
-            ei[j] = be;
-            ev[j] = expf(bv - mx);
-            kept += ev[j];
-            pv = bv;
-            pe = be;
-        }
-        const long long base = ((long long)t * N + n0 + r) * p.k;
-#pragma unroll
-        for (int j = 0; j < 8; ++j)
-            if (j < p.k) {
-                out_idx[base + j] = ei[j];
-                out_gate[base + j] = renorm ? ev[j] / kept : ev[j] / sum;
-            }
-    }
+    for (int r = threadIdx.x; r < ntok; r += nthreads)
+        topk_row(p, lg + r * ldl, (long long)t * p.N + n0 + r, out_idx, out_gate);
 }
 
 // SIMT router for fp32 tokens (or given logits): ECH experts per pass, TOK
