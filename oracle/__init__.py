@@ -20,6 +20,8 @@ Parity status (what pins each function, see ``tests/test_oracle_pins.py``):
                   C=N) and central finite differences of the composed forward
   router_bwd      torch float64 autograd of the whole routed layer (routing fixed,
                   gates differentiable) and central finite differences
+  plan_slices     (planner.py, plain Python) brute-force subset enumeration, a
+                  textbook knapsack instance, equal-weight closed forms
 """
 from __future__ import annotations
 
@@ -29,6 +31,8 @@ import subprocess
 import threading
 
 import numpy as np
+
+from .planner import plan_slices  # noqa: F401  (cross-task slice planner, Section 3.2.1)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "vmoe_oracle.c")
