@@ -223,6 +223,25 @@ int vmoe_router_bwd(const vmoe_problem *p, const void *x, const float *w_router,
                     float *dlogits, float *dw_router, float *dbias, void *dx,
                     void *cuda_stream);
 
+/* Cross-task slice planner (Section 3.2.1, fragmentation-aware expert
+ * grouping; host code, no GPU).  Items (experts) i = 0..n-1 have a memory
+ * footprint weight[i] >= 0 and a lifespan lifespan[i]; the value of an item is
+ * v_i = weight[i] / M - eta * lifespan[i], M = budget if budget > 0, else
+ * capacity.  A 0/1-knapsack DP, dp[i][j] = max(dp[i-1][j], dp[i-1][j - w_i] +
+ * v_i), picks the slice of largest total value whose weight fits `capacity`;
+ * the chosen items leave and the DP runs again until every item is placed.
+ * Items enter the DP in shortest-job-first order (lifespan, then index) and
+ * keep that order inside a slice; an item is taken only when strictly better;
+ * if nothing is chosen, the first remaining item forms a slice alone;
+ * zero-weight items join the first slice.
+ * Output: order[n], the items slice by slice; slice_start[n + 1], where slice s
+ * is order[slice_start[s] .. slice_start[s + 1]).  Returns the number of slices,
+ * VMOE_ERR_INVALID (null pointers, negative weight, NaN lifespan) or
+ * VMOE_ERR_UNSUPPORTED (an item heavier than capacity, or a DP table above 2^30
+ * entries). */
+int vmoe_plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity,
+                     double eta, double budget, int32_t *order, int32_t *slice_start);
+
 /* Device status word of the current device: 0 when clean, otherwise a
  * vmoe_status (VMOE_ERR_DEVICE_TIMEOUT after a kernel gave up a bounded
  * wait).  Synchronises the current device.  `reset` != 0 clears the word. */

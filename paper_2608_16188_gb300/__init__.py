@@ -34,7 +34,7 @@ VMOE_GELU_TANH = 1 << 2
 # Every symbol include/vmoe.h declares.
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
-           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd",
+           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd", "vmoe_plan_slices",
            "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
            "vmoe_trace_disable", "vmoe_trace_get")
 
@@ -79,6 +79,8 @@ def library():
             "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
             "vmoe_router_bwd": (ctypes.c_int, [PP] + [_P] * 13 + [_P]),
+            "vmoe_plan_slices": (ctypes.c_int, [ctypes.c_int, _P, _P, ctypes.c_int64,
+                                                ctypes.c_double, ctypes.c_double, _P, _P]),
             "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
             "vmoe_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_longlong, _P]),
             "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
@@ -197,6 +199,21 @@ def vmoe_router_bwd(p, x, w_router, logits, expert_idx, gate, slot, dy, ye, dgat
         ctypes.byref(p), _ptr(x), _ptr(w_router), _ptr(logits), _ptr(expert_idx), _ptr(gate),
         _ptr(slot), _ptr(dy), _ptr(ye), _ptr(dgate), _ptr(dlogits), _ptr(dw_router), _ptr(dbias),
         _ptr(dx), _stream(stream)), "vmoe_router_bwd")
+
+
+def vmoe_plan_slices(weight, lifespan, capacity: int, eta: float = 0.0, budget: float = 0.0):
+    """Host-side slice planner (see include/vmoe.h); returns a list of slices,
+    each a list of item indices."""
+    import numpy as np
+    w = np.ascontiguousarray(weight, dtype=np.int64)
+    r = np.ascontiguousarray(lifespan, dtype=np.float64)
+    n = int(w.size)
+    order = np.zeros(max(n, 1), dtype=np.int32)
+    start = np.zeros(n + 2, dtype=np.int32)
+    ns = library().vmoe_plan_slices(n, w.ctypes.data, r.ctypes.data, int(capacity), float(eta),
+                                    float(budget), order.ctypes.data, start.ctypes.data)
+    _check(ns if ns < 0 else 0, "vmoe_plan_slices")
+    return [order[start[s]:start[s + 1]].tolist() for s in range(ns)]
 
 
 def vmoe_device_status(reset: bool = False) -> int:

@@ -1,0 +1,99 @@
+// planner.cu -- the cross-task slice planner (host code): Section 3.2.1
+// groups the experts pooled across tasks into ordered time slices that fit a
+// memory budget, by a 0/1-knapsack dynamic programme over each expert's
+// temporary footprint w_i (the weight) and the value
+//     v_i = w_i / M_c - eta * r_i          (r_i: the expert's lifespan),
+//     dp[i][j] = max(dp[i-1][j], dp[i-1][j - w_i] + v_i),
+// run again over the experts left until all are placed.  The library uses it to
+// run the expert backward in slices whose dH fits a caller's workspace.
+//
+// Readings: the experts enter the DP in shortest-job-first order (lifespan,
+// then index), the paper's SJF bias, and keep that order inside a slice;
+// dp[0][j] = 0 for all j (capacity used at most j), an expert is taken only
+// when that is strictly better; an empty choice while experts remain places
+// the first remaining expert alone; zero-footprint experts join the first
+// slice; an expert heavier than the budget is refused.
+#include <stdint.h>
+
+#include <algorithm>
+#include <numeric>
+#include <vector>
+
+#include "vmoe.h"
+
+namespace vmoe {
+
+int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
+                double budget, int32_t *order, int32_t *slice_start) {
+    if (n < 0 || capacity < 0 || (n > 0 && (!weight || !lifespan || !order || !slice_start)))
+        return VMOE_ERR_INVALID;
+    if (!slice_start) return VMOE_ERR_INVALID;
+    for (int i = 0; i < n; ++i) {
+        if (weight[i] < 0 || !(lifespan[i] == lifespan[i])) return VMOE_ERR_INVALID;
+        if (weight[i] > capacity) return VMOE_ERR_UNSUPPORTED;
+    }
+    if (capacity >= (1 << 24) || (int64_t)n * (capacity + 1) > ((int64_t)1 << 30))
+        return VMOE_ERR_UNSUPPORTED;  // DP table too large
+    const int cap = (int)capacity;
+    const double mc = budget > 0.0 ? budget : (double)capacity;
+    std::vector<double> v(n);
+    for (int i = 0; i < n; ++i) v[i] = (mc > 0.0 ? (double)weight[i] / mc : 0.0) - eta * lifespan[i];
+    std::vector<int> sjf(n);
+    std::iota(sjf.begin(), sjf.end(), 0);
+    std::stable_sort(sjf.begin(), sjf.end(), [&](int a, int b) { return lifespan[a] < lifespan[b]; });
+    std::vector<int> zero, remaining;
+    for (int i : sjf) (weight[i] == 0 ? zero : remaining).push_back(i);
+
+    std::vector<std::vector<int>> slices;
+    std::vector<double> dp(cap + 1);
+    std::vector<uint8_t> take;
+    while (!remaining.empty()) {
+        const int m = (int)remaining.size();
+        std::fill(dp.begin(), dp.end(), 0.0);
+        take.assign((size_t)m * (cap + 1), 0);
+        for (int a = 0; a < m; ++a) {
+            const int i = remaining[a];
+            const int wi = (int)weight[i];
+            uint8_t *t = take.data() + (size_t)a * (cap + 1);
+            for (int j = cap; j >= wi; --j) {  // descending: dp[j - wi] is still row a-1
+                const double cand = dp[j - wi] + v[i];
+                if (cand > dp[j]) {
+                    dp[j] = cand;
+                    t[j] = 1;
+                }
+            }
+        }
+        std::vector<uint8_t> chosen(n, 0);
+        int nchosen = 0;
+        for (int a = m - 1, j = cap; a >= 0; --a)
+            if (take[(size_t)a * (cap + 1) + j]) {
+                chosen[remaining[a]] = 1;
+                ++nchosen;
+                j -= (int)weight[remaining[a]];
+            }
+        if (nchosen == 0) chosen[remaining[0]] = 1;
+        std::vector<int> slice, rest;
+        for (int i : remaining) (chosen[i] ? slice : rest).push_back(i);
+        slices.push_back(std::move(slice));
+        remaining.swap(rest);
+    }
+    if (!zero.empty()) {
+        if (slices.empty()) slices.push_back({});
+        slices[0].insert(slices[0].begin(), zero.begin(), zero.end());
+    }
+    int pos = 0;
+    for (size_t s = 0; s < slices.size(); ++s) {
+        slice_start[s] = pos;
+        for (int i : slices[s]) order[pos++] = i;
+    }
+    slice_start[slices.size()] = pos;
+    return (int)slices.size();
+}
+
+}  // namespace vmoe
+
+extern "C" int vmoe_plan_slices(int n, const int64_t *weight, const double *lifespan,
+                                int64_t capacity, double eta, double budget, int32_t *order,
+                                int32_t *slice_start) {
+    return vmoe::plan_slices(n, weight, lifespan, capacity, eta, budget, order, slice_start);
+}
