@@ -148,6 +148,12 @@ int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const
  * its bf16 residual so the weight gradients of small groups stay accurate. */
 size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p);
 
+/* The smallest workspace vmoe_expert_bwd accepts for `p`, or 0 if `p` is
+ * invalid.  Host only.  fp32: the full size above.  bf16: one group's dH (2C
+ * rows, rounded up to 8) plus 8*T*E bytes (rounded up to 256) for the plan of a
+ * sliced run -- see vmoe_expert_bwd. */
+size_t vmoe_expert_bwd_min_workspace_size(const vmoe_problem *p);
+
 /* Expert FFN backward (adaptation of the expert weights, Section 3.1), the
  * gradient of <dY, y> through the expert path with routing and gates fixed:
  *   dH = (dYe W2^T) * GELU'(H), dXe = dH W1^T, dW1 = Xe^T dH, dW2 = A^T dYe,
@@ -156,9 +162,15 @@ size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p);
  *   (= vmoe_dispatch(dY, gate)), load [T,E]
  *   dxe [T,E,C,d] out (rows >= load not written), dw1 [T,E,d,f] out, dw2 [T,E,f,d] out
  *   (every element written; zero for a group with load 0)
- *   workspace: caller-owned device scratch of at least
- *   vmoe_expert_bwd_workspace_size(p) bytes, 16-byte aligned; its contents are
- *   clobbered.  Too small or NULL returns VMOE_ERR_INVALID. */
+ *   workspace: caller-owned device scratch, 16-byte aligned, its contents
+ *   clobbered.  With vmoe_expert_bwd_workspace_size(p) bytes or more, dH of
+ *   every group fits and the call is asynchronous.  bf16 problems also accept
+ *   less, down to vmoe_expert_bwd_min_workspace_size(p): the groups are then
+ *   placed in slices whose dH fits (the cross-task DP of vmoe_plan_slices,
+ *   Section 3.2.1, each group's footprint its dH rows, its lifespan its load)
+ *   and dA, dX and dW1 run slice by slice.  That path reads `load` back to the
+ *   host first and synchronises `cuda_stream`.  The results are bitwise the
+ *   same either way.  Less than the minimum, or NULL, returns VMOE_ERR_INVALID. */
 int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,
                     const void *w1, const void *w2, const void *dye, const int32_t *load,
                     void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,

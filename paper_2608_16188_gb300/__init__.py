@@ -34,6 +34,7 @@ VMOE_GELU_TANH = 1 << 2
 # Every symbol include/vmoe.h declares.
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
+           "vmoe_expert_bwd_min_workspace_size",
            "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd", "vmoe_plan_slices",
            "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
            "vmoe_trace_disable", "vmoe_trace_get")
@@ -75,6 +76,7 @@ def library():
             "vmoe_dispatch": (ctypes.c_int, [PP] + [_P] * 6 + [_P]),
             "vmoe_expert_fwd": (ctypes.c_int, [PP] + [_P] * 7 + [_P]),
             "vmoe_expert_bwd_workspace_size": (ctypes.c_size_t, [PP]),
+            "vmoe_expert_bwd_min_workspace_size": (ctypes.c_size_t, [PP]),
             "vmoe_expert_bwd": (ctypes.c_int, [PP] + [_P] * 11 + [ctypes.c_size_t, _P]),
             "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
@@ -146,6 +148,10 @@ def vmoe_problem_capacity(p: VmoeProblem) -> int:
 
 def vmoe_expert_bwd_workspace_size(p: VmoeProblem) -> int:
     return int(library().vmoe_expert_bwd_workspace_size(ctypes.byref(p)))
+
+
+def vmoe_expert_bwd_min_workspace_size(p: VmoeProblem) -> int:
+    return int(library().vmoe_expert_bwd_min_workspace_size(ctypes.byref(p)))
 
 
 def vmoe_route(p, x, w_router, logit_bias, logits, expert_idx, gate, slot, load, stream=None):

@@ -223,6 +223,12 @@ size_t vmoe_expert_bwd_workspace_size(const vmoe_problem *p) {
     return (size_t)d.T * d.E * d.C * d.f * per_elem;
 }
 
+size_t vmoe_expert_bwd_min_workspace_size(const vmoe_problem *p) {
+    Dims d;
+    if (check_problem(p, &d) != VMOE_OK) return 0;
+    return d.bf16 ? bwd_min_workspace(d) : vmoe_expert_bwd_workspace_size(p);
+}
+
 int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,
                     const void *w1, const void *w2, const void *dye, const int32_t *load,
                     void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,
@@ -234,8 +240,16 @@ int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const 
     if (!dev_ok(xe) || !dev_ok(h) || !dev_ok(a) || !dev_ok(w1) || !dev_ok(w2) || !dev_ok(dye) ||
         !dev_ok(load) || !dev_ok(dxe) || !dev_ok(dw1) || !dev_ok(dw2) || !dev_ok(workspace))
         return VMOE_ERR_INVALID;
-    if (workspace_bytes < vmoe_expert_bwd_workspace_size(p)) return VMOE_ERR_INVALID;
     cudaStream_t s = (cudaStream_t)cuda_stream;
+    if (workspace_bytes < vmoe_expert_bwd_workspace_size(p)) {
+        // a smaller workspace: the backward in slices (bf16 only)
+        if (!d.bf16 || workspace_bytes < bwd_min_workspace(d)) return VMOE_ERR_INVALID;
+        return launch_expert_bwd_bf16_sliced(
+            d, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)h, (const __nv_bfloat16 *)a,
+            (const __nv_bfloat16 *)w1, (const __nv_bfloat16 *)w2, (const __nv_bfloat16 *)dye, load,
+            (__nv_bfloat16 *)dxe, (__nv_bfloat16 *)dw1, (__nv_bfloat16 *)dw2, workspace,
+            workspace_bytes, s, nullptr);
+    }
     if (d.bf16)
         return launch_expert_bwd_bf16(
             d, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)h, (const __nv_bfloat16 *)a,

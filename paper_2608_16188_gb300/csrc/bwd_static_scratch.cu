@@ -8,6 +8,9 @@
 // certified once).  This entry point gives them the same backward with its
 // scratch in a fixed array that lives in the library itself.
 //
+// When dH for every group does not fit, the bf16 backward runs in slices of
+// groups planned to fit the array (vmoe_expert_bwd with a smaller workspace).
+//
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds VMOE_STATIC_SCRATCH_BYTES of it until the process exits.  In
 // host code its name is only a host-side stand-in, so the device address is
@@ -28,7 +31,9 @@ extern "C" int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void 
                                               const void *a, const void *w1, const void *w2,
                                               const void *dye, const int32_t *load, void *dxe,
                                               void *dw1, void *dw2, void *cuda_stream) {
-    const size_t need = vmoe_expert_bwd_workspace_size(p);
+    // dH for every group, or -- bf16 -- at least one group's, which runs the
+    // backward in slices planned to fit the array
+    const size_t need = vmoe_expert_bwd_min_workspace_size(p);
     if (need == 0) return VMOE_ERR_INVALID;                       // invalid problem statement
     if (need > VMOE_STATIC_SCRATCH_BYTES) return VMOE_ERR_UNSUPPORTED;  // too large for the array
     int dev = 0;

@@ -51,6 +51,16 @@ int launch_expert_bwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bf
                            const __nv_bfloat16 *w2, const __nv_bfloat16 *dye,
                            const int32_t *load, __nv_bfloat16 *dxe, __nv_bfloat16 *dw1,
                            __nv_bfloat16 *dw2, __nv_bfloat16 *dh, cudaStream_t s);
+// The expert backward under a dH budget (gemm_tc_bwd.cu): slices planned by
+// the cross-task DP; `workspace` holds the plan, then the slices' dH.
+size_t bwd_plan_bytes(const Dims &p);
+size_t bwd_min_workspace(const Dims &p);
+int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const __nv_bfloat16 *h,
+                                  const __nv_bfloat16 *act, const __nv_bfloat16 *w1,
+                                  const __nv_bfloat16 *w2, const __nv_bfloat16 *dye,
+                                  const int32_t *load, __nv_bfloat16 *dxe, __nv_bfloat16 *dw1,
+                                  __nv_bfloat16 *dw2, void *workspace, size_t workspace_bytes,
+                                  cudaStream_t s, int *nslices_out);
 int launch_router_bwd(const Dims &p, const void *x, const float *w_router, const float *logits,
                       const int32_t *idx, const float *gate, const int32_t *slot, const void *dy,
                       const void *ye, float *dgate, float *dlogits, float *dw_router, float *dbias,

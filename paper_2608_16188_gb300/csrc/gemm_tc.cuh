@@ -96,7 +96,17 @@ struct Args {
     int ksplit;                // weight-gradient mode: B holds [hi rows; lo rows] (K doubled)
     int gelu_tanh;
     int *status;
+    // Slices (the memory-budgeted backward): the launch covers G entries, entry i
+    // being group glist[i] of the real tensors (glist NULL: entry i = group i).
+    // Operands flagged in `compact` live in a compact buffer instead, entry i's
+    // rows starting at row crow[i] (with ksplit / a second output, the residual
+    // rows follow the entry's load rows).
+    const int32_t *glist;
+    const int32_t *crow;
+    int compact;               // CMP_* bits
 };
+enum { CMP_A = 1, CMP_B = 2, CMP_D = 4 };
+__device__ __forceinline__ int real_group(const Args &a, int i) { return a.glist ? __ldg(a.glist + i) : i; }
 
 // ---------------------------------------------------------------------------
 // PTX wrappers.
@@ -274,6 +284,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16(int M, int N, bool a_mn, bool 
 struct Tile {
     int g, m_blk, n_blk, kblocks, kvalid, rows_valid;
     int khalf;  // weight-gradient mode: k-blocks per half (kblocks = 2 * khalf with ksplit)
+    int gr;     // the real group of entry g
+    int crow;   // entry g's first row in the compact buffer
 };
 
 template <int MODE>
@@ -286,20 +298,24 @@ __device__ __forceinline__ Tile decode_tile(const Args &a, const int *prefix, in
             if (prefix[mid] <= u) lo = mid; else hi = mid;
         }
         t.g = lo;
+        t.gr = real_group(a, lo);
+        t.crow = a.crow ? __ldg(a.crow + lo) : 0;
         int local = u - prefix[lo];
         t.m_blk = local / a.tiles_n;
         t.n_blk = local - t.m_blk * a.tiles_n;
         t.kblocks = a.K_fixed / BK;
         t.kvalid = a.K_fixed;
-        int L = __ldg(a.load + t.g);
+        int L = __ldg(a.load + t.gr);
         t.rows_valid = L < 0 ? 0 : (L > a.C ? a.C : L);
     } else {
         int tpg = a.tiles_m * a.tiles_n;
         t.g = u / tpg;
+        t.gr = real_group(a, t.g);
+        t.crow = a.crow ? __ldg(a.crow + t.g) : 0;
         int local = u - t.g * tpg;
         t.m_blk = local / a.tiles_n;
         t.n_blk = local - t.m_blk * a.tiles_n;
-        int L = __ldg(a.load + t.g);
+        int L = __ldg(a.load + t.gr);
         L = L < 0 ? 0 : (L > a.C ? a.C : L);
         t.kvalid = L;
         t.khalf = (L + BK - 1) / BK;
@@ -365,7 +381,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         const int g0 = min(G, tid * per), g1 = min(G, g0 + per);
         int local = 0;
         for (int g = g0; g < g1; ++g) {
-            int L = __ldg(args.load + g);
+            int L = __ldg(args.load + real_group(args, g));
             L = L < 0 ? 0 : (L > args.C ? args.C : L);
             local += ((L + BM - 1) / BM) * args.tiles_n;
         }
@@ -397,7 +413,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         int run = scan_tmp[tid];
         for (int g = g0; g < g1; ++g) {
             prefix[g] = run;
-            int L = __ldg(args.load + g);
+            int L = __ldg(args.load + real_group(args, g));
             L = L < 0 ? 0 : (L > args.C ? args.C : L);
             run += ((L + BM - 1) / BM) * args.tiles_n;
         }
@@ -430,11 +446,14 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const uint32_t fb = bar_full(stage);
                     if (MODE == MODE_ROW) {
                         mbar_expect_tx(fb, S::STAGE_BYTES);
-                        tma_load_3d(sa, &tmA, fb, kb * BK, t.m_blk * BM, t.g);
+                        if (args.compact & CMP_A)
+                            tma_load_3d(sa, &tmA, fb, kb * BK, t.crow + t.m_blk * BM, 0);
+                        else
+                            tma_load_3d(sa, &tmA, fb, kb * BK, t.m_blk * BM, t.gr);
                         if (B_MN) {  // one 4-D box: BN/64 column chunks of 64 rows
-                            tma_load_4d(sb, &tmB, fb, 0, kb * BK, t.n_blk * (BN / 64), t.g);
+                            tma_load_4d(sb, &tmB, fb, 0, kb * BK, t.n_blk * (BN / 64), t.gr);
                         } else {
-                            tma_load_3d(sb, &tmB, fb, kb * BK, t.n_blk * BN, t.g);
+                            tma_load_3d(sb, &tmB, fb, kb * BK, t.n_blk * BN, t.gr);
                         }
                     } else {
                         // Weight gradients: K = the group's rows.  With ksplit the second
@@ -444,8 +463,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                         const int hi = (kb >= t.khalf) ? 1 : 0;
                         const int ka = (kb - hi * t.khalf) * BK;
                         const int kbr = hi * args.C + ka;
-                        tma_load_4d(sa, &tmA, fb, 0, ka, t.m_blk * (BM / 64), t.g);
-                        tma_load_4d(sb, &tmB, fb, 0, kbr, t.n_blk * (BN / 64), t.g);
+                        tma_load_4d(sa, &tmA, fb, 0, ka, t.m_blk * (BM / 64), t.gr);
+                        if (args.compact & CMP_B)  // residual rows follow the entry's load rows
+                            tma_load_4d(sb, &tmB, fb, 0, t.crow + hi * t.kvalid + ka,
+                                        t.n_blk * (BN / 64), 0);
+                        else
+                            tma_load_4d(sb, &tmB, fb, 0, kbr, t.n_blk * (BN / 64), t.gr);
                     }
                     issued[stage]++;
                     if (++stage == STAGES) {
@@ -596,7 +619,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 fence_proxy_async();
                 __syncwarp();
                 if (lane == 0) {
-                    tma_store_3d(&tmD, smem_u32(buf), colw + c * 64, row0, t.g);
+                    tma_store_3d(&tmD, smem_u32(buf), colw + c * 64, row0, t.gr);
                     bulk_commit();
                 }
                 ++nstore;
@@ -628,7 +651,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int r0 = tl.m_blk * BM + q * 32;
             if (r0 + lane < tl.rows_valid) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
-                    args.aux + (long long)tl.g * args.sAux + (long long)(r0 + lane) * args.ldd +
+                    args.aux + (long long)tl.gr * args.sAux + (long long)(r0 + lane) * args.ldd +
                     tl.n_blk * BN + half * COLS + sc * 32);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
@@ -681,7 +704,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             int nvalid = t.rows_valid - row0;
             nvalid = nvalid < 0 ? 0 : (nvalid > 32 ? 32 : nvalid);
             const int colw = t.n_blk * BN + half * COLS;
-            const long long gofs = (long long)t.g * args.sD + (long long)row0 * args.ldd + colw;
+            const long long gofs = (long long)t.gr * args.sD + (long long)row0 * args.ldd + colw;
             const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
                                   (uint32_t)(acc * BN + half * COLS);
             uint8_t *bufD = stg, *bufA = stg + 4096;
@@ -732,10 +755,10 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     }
                     if ((sc & 1) == 1) {
                         const int c64 = (sc >> 1) * 64;
-                        flush(bufD, &tmD, args.D + gofs + c64, colw + c64, row0, t.g, nvalid);
+                        flush(bufD, &tmD, args.D + gofs + c64, colw + c64, row0, t.gr, nvalid);
                         ++nstore;
                         if (NOUT == 2) {
-                            flush(bufA, &tmD2, args.D2 + gofs + c64, colw + c64, row0, t.g, nvalid);
+                            flush(bufA, &tmD2, args.D2 + gofs + c64, colw + c64, row0, t.gr, nvalid);
                             ++nstore;
                         }
                     }
@@ -773,7 +796,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int r0 = tl.m_blk * BM + q * 32;
             if (r0 + lane < tl.rows_valid) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
-                    args.aux + (long long)tl.g * args.sAux + (long long)(r0 + lane) * args.ldd +
+                    args.aux + (long long)tl.gr * args.sAux + (long long)(r0 + lane) * args.ldd +
                     tl.n_blk * BN + half * COLS + c * 32);
 #pragma unroll
                 for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
@@ -808,8 +831,12 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             const int row0 = t.m_blk * BM + q * 32;  // this warp's first row in the group
             int nvalid = t.rows_valid - row0;
             nvalid = nvalid < 0 ? 0 : (nvalid > 32 ? 32 : nvalid);
-            const long long gofs = (long long)t.g * args.sD + (long long)row0 * args.ldd +
-                                   t.n_blk * BN + half * COLS;
+            // compact output: the entry's rows from crow, its second output (the
+            // residual) after its load rows; else the group's slab
+            const bool cmpd = (args.compact & CMP_D) != 0;
+            const long long gofs = (cmpd ? (long long)t.crow * args.ldd : (long long)t.gr * args.sD) +
+                                   (long long)row0 * args.ldd + t.n_blk * BN + half * COLS;
+            const long long gofs2 = cmpd ? gofs + (long long)t.rows_valid * args.ldd : gofs;
             const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
                                   (uint32_t)(acc * BN + half * COLS);
             for (int c = 0; c < NCH; ++c) {
@@ -853,7 +880,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                             }
                             *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(lv);
                         }
-                        store_rows(args.D2 + gofs + c * 32, nvalid);
+                        store_rows(args.D2 + gofs2 + c * 32, nvalid);
                     }
                     if (EPI == EPI_GELU) {
 #pragma unroll
@@ -863,7 +890,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                             for (int e = 0; e < 8; ++e) gv[e] = gelu_fast(v[i * 8 + e], tanh_form);
                             *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(gv);
                         }
-                        store_rows(args.D2 + gofs + c * 32, nvalid);
+                        store_rows(args.D2 + gofs2 + c * 32, nvalid);
                     }
                 }
                 if (EPI == EPI_DGELU) {
@@ -980,10 +1007,14 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     const uint32_t tmem_base = (uint32_t)misc[0];
     const int nch = (args.tiles_m + S::MCH - 1) / S::MCH;
     const int total = args.G * args.tiles_n * nch;
-    // unit u -> group, column tile, first row tile and row-tile count
+    // unit u -> entry (its real group g and compact row crow), column tile,
+    // first row tile and row-tile count
+    int crow = 0;
     auto decode = [&](int u, int &g, int &n_blk, int &m0, int &mcnt, int &L) {
-        g = u / (args.tiles_n * nch);
-        const int r = u - g * args.tiles_n * nch;
+        const int i = u / (args.tiles_n * nch);
+        const int r = u - i * args.tiles_n * nch;
+        g = real_group(args, i);
+        crow = args.crow ? __ldg(args.crow + i) : 0;
         n_blk = r / nch;
         m0 = (r - n_blk * nch) * S::MCH;
         mcnt = min(S::MCH, args.tiles_m - m0);
@@ -1009,12 +1040,14 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                     break;
                 const uint32_t bdst = smem_u32(b_res) + bb * S::B_BYTES;
                 mbar_expect_tx(bar_bfull(bb), (uint32_t)(nkb * (KSPLIT ? 2 : 1)) * S::B_KB);
+                const bool cmpb = (args.compact & CMP_B) != 0;  // B rows from crow, residual after L
                 for (int kb = 0; kb < nkb; ++kb) {
-                    tma_load_4d(bdst + kb * S::B_KB, &tmB, bar_bfull(bb), 0, kb * BK,
-                                n_blk * (BN / 64), g);
+                    tma_load_4d(bdst + kb * S::B_KB, &tmB, bar_bfull(bb), 0,
+                                (cmpb ? crow : 0) + kb * BK, n_blk * (BN / 64), cmpb ? 0 : g);
                     if (KSPLIT)
                         tma_load_4d(bdst + (2 + kb) * S::B_KB, &tmB, bar_bfull(bb), 0,
-                                    args.C + kb * BK, n_blk * (BN / 64), g);
+                                    (cmpb ? crow + L : args.C) + kb * BK, n_blk * (BN / 64),
+                                    cmpb ? 0 : g);
                 }
                 ++b_issued[bb];
                 ++ub;
@@ -1277,6 +1310,18 @@ int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap
     return launch_result();
 }
 
+// A slice of the groups for one launch (the memory-budgeted backward): n
+// entries, entry i = group glist[i]; the operands flagged in `compact` live in
+// a compact buffer of `rows` rows, entry i's rows from crow[i].  n == 0: all
+// groups, nothing compact.
+struct Slice {
+    const int32_t *glist = nullptr;  // device
+    const int32_t *crow = nullptr;   // device
+    int n = 0;
+    int compact = 0;
+    long long rows = 0;
+};
+
 inline Args base_args(const Dims &p, const int32_t *load) {
     Args a = {};
     a.G = p.G();
@@ -1295,12 +1340,14 @@ template <int EPI, bool B_MN>
 int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16 *w, int N,
              const int32_t *load, __nv_bfloat16 *D, __nv_bfloat16 *D2, const __nv_bfloat16 *aux,
              cudaStream_t s, const char *name, long long sD = 0, long long sAux = 0,
-             long long sAct = 0) {
+             long long sAct = 0, const Slice &sl = Slice()) {
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
     CUtensorMap ma, mb;
-    if (!make_map(&ma, act, K, C, G, 128, (uint64_t)sAct)) return VMOE_ERR_CUDA;
+    const bool okA = (sl.compact & CMP_A) ? make_map(&ma, act, K, (uint64_t)sl.rows, 1, 128)
+                                          : make_map(&ma, act, K, C, G, 128, (uint64_t)sAct);
+    if (!okA) return VMOE_ERR_CUDA;
     bool okb = B_MN ? make_map_chunked(&mb, w, N, K, G, 64, BN / 64) : make_map(&mb, w, K, N, G, BN);
     if (!okb) return VMOE_ERR_CUDA;
     Args a = base_args(p, load);
@@ -1314,7 +1361,13 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
     a.sD = sD ? sD : (long long)C * N;
     a.sAux = sAux ? sAux : (long long)C * N;
     a.ldd = N;
-    long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
+    if (sl.n > 0) {
+        a.G = sl.n;
+        a.glist = sl.glist;
+        a.crow = sl.crow;
+        a.compact = sl.compact;
+    }
+    long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
     CUtensorMap md = {}, md2 = {};  // output maps: 64 x 32 store boxes over [G, C, N]
     if (UseTmaStore<MODE_ROW, EPI>::value) {
         if (!make_map(&md, D, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
@@ -1330,13 +1383,17 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
 // rows [C, 2C) -- and D = act1^T (hi + lo), the K loop running over both halves.
 inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __nv_bfloat16 *act2,
                       int N, const int32_t *load, __nv_bfloat16 *D, cudaStream_t s,
-                      const char *name, bool ksplit = false) {
+                      const char *name, bool ksplit = false, const Slice &sl = Slice()) {
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
+    const bool cmpb = (sl.compact & CMP_B) != 0;
+    // B: per-group slabs of C (with ksplit 2C) rows, or the compact buffer
+    const uint64_t b_rows = cmpb ? (uint64_t)sl.rows : (uint64_t)(ksplit ? 2 * C : C);
+    const uint64_t b_outer = cmpb ? 1 : (uint64_t)G;
     CUtensorMap ma, mb, md;
     if (!make_map_chunked(&ma, act1, M, C, G, 64, BM / 64)) return VMOE_ERR_CUDA;
-    if (!make_map_chunked(&mb, act2, N, ksplit ? 2 * C : C, G, 64, BN / 64)) return VMOE_ERR_CUDA;
+    if (!make_map_chunked(&mb, act2, N, b_rows, b_outer, 64, BN / 64)) return VMOE_ERR_CUDA;
     if (!make_map(&md, D, N, M, G, 32)) return VMOE_ERR_CUDA;  // 64 x 32 store boxes
     Args a = base_args(p, load);
     a.N = N;
@@ -1347,16 +1404,22 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     a.sD = (long long)M * N;
     a.ldd = N;
     a.ksplit = ksplit ? 1 : 0;
+    if (sl.n > 0) {
+        a.G = sl.n;
+        a.glist = sl.glist;
+        a.crow = sl.crow;
+        a.compact = sl.compact;
+    }
     if (ksplit && N % BSTAT_BN == 0 && C <= 2 * BK) {  // every group fits one resident B tile
         using SB = BStatShape<BSTAT_BN, true, BSTAT_BUFS>;
         CUtensorMap mbs;
-        if (!make_map_chunked(&mbs, act2, N, 2 * C, G, 64, BSTAT_BN / 64)) return VMOE_ERR_CUDA;
+        if (!make_map_chunked(&mbs, act2, N, b_rows, b_outer, 64, BSTAT_BN / 64)) return VMOE_ERR_CUDA;
         a.tiles_n = N / BSTAT_BN;
         const int nch = (a.tiles_m + SB::MCH - 1) / SB::MCH;
-        const long long units = (long long)G * a.tiles_n * nch;
+        const long long units = (long long)a.G * a.tiles_n * nch;
         return launch_bstat<BSTAT_BN, true, BSTAT_BUFS>(ma, mbs, md, a, units, s, name);
     }
-    long long max_tiles = (long long)G * a.tiles_m * a.tiles_n;
+    long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
     return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name)
                 : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name);
 }

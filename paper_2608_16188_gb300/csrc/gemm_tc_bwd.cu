@@ -3,9 +3,14 @@
 //   dX:         dXe = dH W1^T               (A: dH K-major;  B: W1 [d,f] read K-major)
 //   dW1:        dW1 = Xe^T dH               (both MN-major, K = load)
 //   dW2:        dW2 = A^T dYe               (both MN-major, K = load)
+#include <vector>
+
 #include "gemm_tc.cuh"
 
 namespace vmoe {
+
+int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
+                double budget, int32_t *order, int32_t *slice_start);  // planner.cu
 
 using namespace tc;
 
@@ -28,6 +33,89 @@ int launch_expert_bwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bf
         return st;
     if ((st = wgrad_gemm(p, xe, p.d, dh, p.f, load, dw1, s, "tc_dw1", true)) != VMOE_OK) return st;
     return wgrad_gemm(p, act, p.f, dye, p.d, load, dw2, s, "tc_dw2");
+}
+
+// The backward under a dH budget (the expert groups' temporary memory, Section
+// 3.2.1): when the workspace cannot hold dH for every group, the groups are
+// placed in slices by the cross-task DP planner, each group's footprint being
+// its dH rows (load rows of dH_hi, then load rows of the residual), in units of
+// BW_UNIT rows; the slice's groups are packed into the workspace at 8-row
+// offsets, and dA, dX and dW1 run per slice.  dW2 needs no dH and runs once.
+// The loads are read back to the host first (one stream synchronisation); the
+// plan (group list and first rows) goes to the head of the workspace.
+constexpr int BW_UNIT = 8;
+
+size_t bwd_plan_bytes(const Dims &p) { return (((size_t)2 * p.G() * sizeof(int32_t)) + 255) & ~(size_t)255; }
+
+size_t bwd_min_workspace(const Dims &p) {
+    const size_t unit_rows = ((size_t)2 * p.C + BW_UNIT - 1) / BW_UNIT * BW_UNIT;
+    return bwd_plan_bytes(p) + unit_rows * p.f * sizeof(__nv_bfloat16);
+}
+
+int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const __nv_bfloat16 *h,
+                                  const __nv_bfloat16 *act, const __nv_bfloat16 *w1,
+                                  const __nv_bfloat16 *w2, const __nv_bfloat16 *dye,
+                                  const int32_t *load, __nv_bfloat16 *dxe, __nv_bfloat16 *dw1,
+                                  __nv_bfloat16 *dw2, void *workspace, size_t workspace_bytes,
+                                  cudaStream_t s, int *nslices_out) {
+    const int G = p.G();
+    const size_t plan_bytes = bwd_plan_bytes(p);
+    if (workspace_bytes < bwd_min_workspace(p)) return VMOE_ERR_INVALID;
+    const long long rows = (long long)((workspace_bytes - plan_bytes) / ((size_t)p.f * sizeof(__nv_bfloat16)));
+    const long long cap_units = rows / BW_UNIT;
+    std::vector<int32_t> hload(G);
+    if (cudaMemcpyAsync(hload.data(), load, sizeof(int32_t) * G, cudaMemcpyDeviceToHost, s) !=
+            cudaSuccess ||
+        cudaStreamSynchronize(s) != cudaSuccess)
+        return VMOE_ERR_CUDA;
+    std::vector<int64_t> w(G);
+    std::vector<double> r(G);
+    for (int g = 0; g < G; ++g) {
+        const int L = hload[g] < 0 ? 0 : (hload[g] > p.C ? p.C : hload[g]);
+        hload[g] = L;
+        w[g] = (2LL * L + BW_UNIT - 1) / BW_UNIT;
+        r[g] = (double)L;
+    }
+    std::vector<int32_t> order(G), start(G + 1);
+    const int ns = plan_slices(G, w.data(), r.data(), cap_units, 0.0, 0.0, order.data(), start.data());
+    if (ns < 0) return ns;
+    // plan on the device: [glist (G)][crow (G)], slice by slice
+    std::vector<int32_t> plan(2 * (size_t)G);
+    for (int sidx = 0; sidx < ns; ++sidx) {
+        long long row = 0;
+        for (int k = start[sidx]; k < start[sidx + 1]; ++k) {
+            plan[k] = order[k];
+            plan[G + k] = (int32_t)row;
+            row += w[order[k]] * BW_UNIT;
+        }
+    }
+    int32_t *dplan = reinterpret_cast<int32_t *>(workspace);
+    __nv_bfloat16 *dh = reinterpret_cast<__nv_bfloat16 *>(static_cast<uint8_t *>(workspace) + plan_bytes);
+    if (cudaMemcpyAsync(dplan, plan.data(), sizeof(int32_t) * 2 * G, cudaMemcpyHostToDevice, s) !=
+        cudaSuccess)
+        return VMOE_ERR_CUDA;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return VMOE_ERR_CUDA;  // host plan buffer is freed on return
+    int st = VMOE_OK;
+    for (int sidx = 0; sidx < ns && st == VMOE_OK; ++sidx) {
+        Slice sl;
+        sl.glist = dplan + start[sidx];
+        sl.crow = dplan + G + start[sidx];
+        sl.n = start[sidx + 1] - start[sidx];
+        sl.rows = rows;
+        sl.compact = CMP_D;
+        st = row_gemm<EPI_DGELU, false>(p, dye, p.d, w2, p.f, load, dh, dh, h, s, "tc_da_dgelu", 0, 0, 0,
+                                        sl);
+        if (st != VMOE_OK) break;
+        sl.compact = CMP_A;
+        st = row_gemm<EPI_STORE, false>(p, dh, p.f, w1, p.d, load, dxe, nullptr, nullptr, s, "tc_dx", 0,
+                                        0, 0, sl);
+        if (st != VMOE_OK) break;
+        sl.compact = CMP_B;
+        st = wgrad_gemm(p, xe, p.d, dh, p.f, load, dw1, s, "tc_dw1", true, sl);
+    }
+    if (st == VMOE_OK) st = wgrad_gemm(p, act, p.f, dye, p.d, load, dw2, s, "tc_dw2");
+    if (nslices_out) *nslices_out = ns;
+    return st;
 }
 
 }  // namespace vmoe

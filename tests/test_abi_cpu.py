@@ -89,15 +89,27 @@ def test_null_and_misaligned_pointers_are_rejected_without_cuda(vm):
     assert st == vm.VMOE_ERR_INVALID  # slot missing
     st = lib.vmoe_expert_fwd(ctypes.byref(p), P, P, P, P, P, P, None, None)
     assert st == vm.VMOE_ERR_INVALID  # ye missing
-    ws = vm.vmoe_expert_bwd_workspace_size(p)
-    st = lib.vmoe_expert_bwd(ctypes.byref(p), P, P, P, P, P, P, P, P, P, P, P, ws - 1, None)
-    assert st == vm.VMOE_ERR_INVALID  # workspace one byte short
+    ws_min = vm.vmoe_expert_bwd_min_workspace_size(p)
+    st = lib.vmoe_expert_bwd(ctypes.byref(p), P, P, P, P, P, P, P, P, P, P, P, ws_min - 1, None)
+    assert st == vm.VMOE_ERR_INVALID  # workspace one byte short of the sliced minimum
+    pf = vm.problem(2, 64, 128, 256, 4, 2, 1.25, "f32")
+    ws = vm.vmoe_expert_bwd_workspace_size(pf)
+    assert vm.vmoe_expert_bwd_min_workspace_size(pf) == ws  # fp32: no sliced path
+    st = lib.vmoe_expert_bwd(ctypes.byref(pf), P, P, P, P, P, P, P, P, P, P, P, ws - 1, None)
+    assert st == vm.VMOE_ERR_INVALID  # fp32 workspace one byte short
     odd = vm.problem(2, 64, 64, 256, 4, 2, 1.25, "bf16")  # bf16 path needs d % 128 == 0
     st = lib.vmoe_expert_fwd(ctypes.byref(odd), P, P, P, P, P, P, P, None)
     assert st == vm.VMOE_ERR_UNSUPPORTED
-    st = lib.vmoe_expert_bwd_static_scratch(ctypes.byref(vm.problem(17, 1576, 768, 3072, 32, 2, 1.25)),
-                                            P, P, P, P, P, P, P, P, P, P, None)
-    assert st == vm.VMOE_ERR_UNSUPPORTED  # dH larger than the static array
+    st = lib.vmoe_expert_bwd_static_scratch(
+        ctypes.byref(vm.problem(17, 1576, 768, 3072, 32, 2, 1.25, "f32")), P, P, P, P, P, P, P, P,
+        P, P, None)
+    assert st == vm.VMOE_ERR_UNSUPPORTED  # fp32 dH larger than the static array (no slices)
+    big = vm.problem(1, 8192, 128, 8192, 1, 1, 1.0)  # one group's dH (2 x 8192 x 8192 bf16) > 64 MiB
+    st = lib.vmoe_expert_bwd_static_scratch(ctypes.byref(big), P, P, P, P, P, P, P, P, P, P, None)
+    assert st == vm.VMOE_ERR_UNSUPPORTED
+    # the 17-task bf16 step fits in slices: one group's dH plus the plan
+    t17 = vm.problem(17, 1576, 768, 3072, 32, 2, 1.25)
+    assert vm.vmoe_expert_bwd_min_workspace_size(t17) == 4352 + 248 * 3072 * 2
     # router backward: W_r is required with dx, logits with VMOE_NO_RENORM
     st = lib.vmoe_router_bwd(ctypes.byref(p), P, None, None, P, P, P, P, P, P, P, P, None, P, None)
     assert st == vm.VMOE_ERR_INVALID
