@@ -314,6 +314,27 @@ def run_ours(args, cfg, rank, world, local_rank):
     if st != 0:
         raise RuntimeError("device status after router backward: " + vm.status_string(st))
 
+    # ---- the expert backward under a 64 MiB dH budget (the static-scratch entry
+    # point, which plans slices with the cross-task DP and synchronises once to
+    # read the loads), against the same backward with a full workspace
+    b = runner.b
+    bw_args = (p, b.xe, b.h, b.a, inp["w1"], inp["w2"], b.dye, b.load, b.dxe, b.dw1, b.dw2)
+    for _ in range(2):
+        vm.vmoe_expert_bwd_static_scratch(*bw_args)
+    torch.cuda.synchronize(dev)
+    bw_calls = 10
+    vm.vmoe_trace_enable(bw_calls * 40 + 16)
+    t0 = time.perf_counter()
+    for _ in range(bw_calls):
+        vm.vmoe_expert_bwd_static_scratch(*bw_args)
+    torch.cuda.synchronize(dev)
+    bw_wall = (time.perf_counter() - t0) / bw_calls
+    n_bw = vm.vmoe_trace_disable()
+    bw_kernel_ms = sum(vm.vmoe_trace_get(i)[1] for i in range(n_bw)) / bw_calls
+    st = vm.vmoe_device_status()
+    if st != 0:
+        raise RuntimeError("device status after the budgeted backward: " + vm.status_string(st))
+
     # ---- max over ranks
     ms_total, e2e_s, e2e_serial_s = max_over_ranks([ms_total, e2e_s, e2e_serial_s], dist, dev)
     tokens_per_step = cfg.T * cfg.N * world
@@ -399,6 +420,18 @@ def run_ours(args, cfg, rank, world, local_rank):
                 "serial_value": round(tokens_per_step * e2e_steps / e2e_serial_s, 1)},
         "clocks": clocks,
         "router_bwd": router_bwd,
+        "budgeted_bwd": {
+            "what": "vmoe_expert_bwd_static_scratch: the expert backward with dH limited to the "
+                    "library's 64 MiB array, groups in slices planned by the cross-task DP",
+            "budget_bytes": vm.VMOE_STATIC_SCRATCH_BYTES,
+            "full_workspace_bytes": vm.vmoe_expert_bwd_workspace_size(p),
+            "ms_per_call_wall": round(bw_wall * 1e3, 4),
+            "kernel_ms_per_call": round(bw_kernel_ms, 4),
+            "launches_per_call": n_bw // bw_calls,
+            "full_workspace_kernel_ms": round(sum(kstats[k]["ms_avg"] for k in
+                                                  ("tc_da_dgelu", "tc_dx", "tc_dw1", "tc_dw2")
+                                                  if k in kstats), 4),
+        },
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(cfg, budget_s=args.cpu_budget)
