@@ -2,6 +2,7 @@
 // rule, dtype selection, the device status word and the kernel trace.
 #include <math.h>
 #include <stdio.h>
+#include <stdlib.h>
 #include <string.h>
 
 #include <vector>
@@ -24,6 +25,14 @@ int *device_status_word() {
         addr[dev] = static_cast<int *>(p);
     }
     return addr[dev];
+}
+
+bool pdl_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("VMOE_PDL");
+        return !(v && v[0] == '0');
+    }();
+    return on;
 }
 
 int num_sms() {

@@ -5,6 +5,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <utility>
+
 #include "vmoe.h"
 
 namespace vmoe {
@@ -27,6 +29,33 @@ int num_sms();              // SM count of the current device
 inline int launch_result() {
     cudaError_t e = cudaGetLastError();
     return e == cudaSuccess ? VMOE_OK : VMOE_ERR_CUDA;
+}
+
+// Programmatic dependent launch for the kernels of a step: each launches with
+// programmatic stream serialisation and waits for its predecessor's results
+// (pdl_wait) only after its own set-up -- barriers, TMEM, tensor-map prefetch.
+// The grouped GEMMs let their successor launch once every CTA has reached its
+// last tile (pdl_launch_dependents); the other kernels at exit.  Letting it
+// launch at the start measured slower: the waiting CTAs of the successor hold
+// warp slots and registers on every SM while the predecessor runs.
+// On by default; the environment variable VMOE_PDL=0 turns it off.
+bool pdl_enabled();  // abi.cu
+
+template <typename... KArgs, typename... Args>
+int launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
+                  Args &&...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    return cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...) == cudaSuccess ? VMOE_OK
+                                                                                    : VMOE_ERR_CUDA;
 }
 
 // Launchers (one file each).
@@ -68,6 +97,13 @@ int launch_router_bwd(const Dims &p, const void *x, const float *w_router, const
 
 // ---------------------------------------------------------------------------
 // Device helpers.
+
+// Programmatic dependent launch (see launch_kernel); both are no-ops in a
+// kernel launched without the attribute.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
 
 // 8 bf16 <-> 8 floats through one 16-byte vector.
 __device__ __forceinline__ void bf16x8_to_f32(const uint4 &v, float *out) {

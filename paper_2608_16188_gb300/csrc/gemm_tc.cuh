@@ -372,6 +372,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         tmem_alloc(smem_u32(misc), S::TMEM_COLS);
         tmem_relinquish();
     }
+    pdl_wait();  // the predecessor's outputs (loads, operands) are complete from here on
 
     // Tile count (and, in row mode, the per-group tile prefix).
     int total;
@@ -436,6 +437,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             bool ok = true;
             for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
                 const Tile t = decode_tile<MODE>(args, prefix, u);
+                if (u + (int)gridDim.x >= total) pdl_launch_dependents();  // this CTA's last tile
                 for (int kb = 0; kb < t.kblocks; ++kb) {
                     if (!wait_phase(bar_empty(stage), phase ^ 1u, abort_flag, args.status)) {
                         ok = false;
@@ -1004,6 +1006,7 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    pdl_wait();  // the predecessor's outputs are complete from here on
     const uint32_t tmem_base = (uint32_t)misc[0];
     const int nch = (args.tiles_m + S::MCH - 1) / S::MCH;
     const int total = args.G * args.tiles_n * nch;
@@ -1032,6 +1035,7 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
             for (int u = blockIdx.x; u < total && ok; u += gridDim.x) {
                 int g, n_blk, m0, mcnt, L;
                 decode(u, g, n_blk, m0, mcnt, L);
+                if (u + (int)gridDim.x >= total) pdl_launch_dependents();  // this CTA's last unit
                 const int nkb = (L + BK - 1) / BK;
                 if (nkb == 0) continue;
                 const int bb = ub % B_BUFS;
@@ -1283,9 +1287,10 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
     if (max_tiles <= 0) return VMOE_OK;
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
-    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, md, md2, a);
+    const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(THREADS), S::SMEM_BYTES, s, ma, mb,
+                                 md, md2, a);
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 template <int BN, bool KSPLIT, int B_BUFS>
@@ -1305,9 +1310,10 @@ int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap
     if (units <= 0) return VMOE_OK;
     long long grid = units < num_sms() ? units : num_sms();
     trace_before(s, name);
-    kern<<<(unsigned)grid, THREADS, S::SMEM_BYTES, s>>>(ma, mb, md, a);
+    const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(THREADS), S::SMEM_BYTES, s, ma, mb,
+                                 md, a);
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 // A slice of the groups for one launch (the memory-budgeted backward): n

@@ -44,6 +44,7 @@ __global__ void __launch_bounds__(PM_THREADS)
 dispatch_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
                 const int32_t *__restrict__ idx, const int32_t *__restrict__ slot,
                 const int32_t *__restrict__ load, T *__restrict__ dst) {
+    pdl_wait();
     constexpr int V = Vec<T>::n;
     const long long row = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -100,6 +101,7 @@ __global__ void __launch_bounds__(PM_THREADS)
 combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
                const int32_t *__restrict__ idx, const int32_t *__restrict__ slot,
                T *__restrict__ dst) {
+    pdl_wait();
     constexpr int V = Vec<T>::n;
     const long long tn = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
     if (tn >= (long long)p.T * p.N) return;
@@ -162,31 +164,32 @@ int launch_dispatch(const Dims &p, const void *src, const float *weight, const i
     long long rows = (long long)p.T * p.N * p.k + (long long)p.T * p.E * p.C;
     long long blocks = (rows + PM_WARPS - 1) / PM_WARPS;
     if (blocks > 0x7fffffffLL) return VMOE_ERR_UNSUPPORTED;
+    int st;
     trace_before(s, "dispatch");
     if (p.bf16)
-        dispatch_kernel<__nv_bfloat16><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+        st = launch_kernel(dispatch_kernel<__nv_bfloat16>, dim3((unsigned)blocks), dim3(PM_THREADS), 0, s,
             p, (const __nv_bfloat16 *)src, weight, idx, slot, load, (__nv_bfloat16 *)dst);
     else
-        dispatch_kernel<float><<<(unsigned)blocks, PM_THREADS, 0, s>>>(
+        st = launch_kernel(dispatch_kernel<float>, dim3((unsigned)blocks), dim3(PM_THREADS), 0, s,
             p, (const float *)src, weight, idx, slot, load, (float *)dst);
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 template <typename T>
-static void combine_as(const Dims &p, const void *src, const float *weight, const int32_t *idx,
+static int combine_as(const Dims &p, const void *src, const float *weight, const int32_t *idx,
                        const int32_t *slot, void *dst, long long blocks, cudaStream_t s) {
     const T *in = (const T *)src;
     T *out = (T *)dst;
     const unsigned nb = (unsigned)blocks;
     if (p.k == 1)
-        combine_kernel<T, 1><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 1>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
     else if (p.k == 2)
-        combine_kernel<T, 2><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 2>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
     else if (p.k <= 4)
-        combine_kernel<T, 4><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 4>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
     else
-        combine_kernel<T, 8><<<nb, PM_THREADS, 0, s>>>(p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 8>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
 }
 
 int launch_combine(const Dims &p, const void *src, const float *weight, const int32_t *idx,
@@ -194,12 +197,10 @@ int launch_combine(const Dims &p, const void *src, const float *weight, const in
     long long rows = (long long)p.T * p.N;
     long long blocks = (rows + PM_WARPS - 1) / PM_WARPS;
     trace_before(s, "combine");
-    if (p.bf16)
-        combine_as<__nv_bfloat16>(p, src, weight, idx, slot, dst, blocks, s);
-    else
-        combine_as<float>(p, src, weight, idx, slot, dst, blocks, s);
+    const int st = p.bf16 ? combine_as<__nv_bfloat16>(p, src, weight, idx, slot, dst, blocks, s)
+                          : combine_as<float>(p, src, weight, idx, slot, dst, blocks, s);
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 }  // namespace vmoe

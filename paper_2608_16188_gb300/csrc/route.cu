@@ -165,6 +165,7 @@ __global__ void __launch_bounds__(RM_THREADS)
 route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__restrict__ wr,
                  const float *__restrict__ bias, float *__restrict__ logits,
                  int32_t *__restrict__ out_idx, float *__restrict__ out_gate) {
+    pdl_wait();
     constexpr int NP = NB * 8;
     constexpr int WP = NP + 8;  // packed-pair row pitch in 32-bit words
     extern __shared__ __align__(16) uint8_t rm_smem[];
@@ -285,9 +286,10 @@ int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, co
     }
     dim3 grid((p.N + RM_TOK - 1) / RM_TOK, p.T);
     trace_before(s, "route_topk");
-    route_mma_kernel<NB><<<grid, RM_THREADS, smem, s>>>(p, x, wr, bias, logits, idx, gate);
+    const int st = launch_kernel(route_mma_kernel<NB>, grid, dim3(RM_THREADS), smem, s, p, x, wr, bias,
+                                 logits, idx, gate);
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 constexpr int CS_THREADS = 256;
@@ -299,6 +301,7 @@ template <bool SMEM_IDX>
 __global__ void __launch_bounds__(CS_THREADS)
 capacity_scan_kernel(Dims p, const int32_t *__restrict__ idx, int32_t *__restrict__ slot,
                      int32_t *__restrict__ load) {
+    pdl_wait();
     extern __shared__ int cs_smem[];
     int *cnt = cs_smem;  // [CS_WARPS][E]
     const int t = blockIdx.x;
@@ -418,12 +421,14 @@ int launch_route(const Dims &p, const void *x, const float *w_router, const floa
                                  cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
             attr_done |= 1ull << dev;
         }
-        capacity_scan_kernel<true><<<p.T, CS_THREADS, smem_big, s>>>(p, idx, slot, load);
+        st = launch_kernel(capacity_scan_kernel<true>, dim3(p.T), dim3(CS_THREADS), smem_big, s, p,
+                           idx, slot, load);
     } else {
-        capacity_scan_kernel<false><<<p.T, CS_THREADS, smem_small, s>>>(p, idx, slot, load);
+        st = launch_kernel(capacity_scan_kernel<false>, dim3(p.T), dim3(CS_THREADS), smem_small, s,
+                           p, idx, slot, load);
     }
     trace_after(s);
-    return launch_result();
+    return st;
 }
 
 }  // namespace vmoe
