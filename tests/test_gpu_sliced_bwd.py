@@ -73,3 +73,25 @@ def test_sliced_backward_rejects_a_workspace_below_the_minimum():
         vm.vmoe_expert_bwd(p, b.xe, b.h, b.a, inp["w1"], inp["w2"], b.dye, b.load, b.dxe, b.dw1,
                            b.dw2, ws)
     assert e.value.status == vm.VMOE_ERR_INVALID
+
+
+def test_sliced_backward_at_the_17_task_step():
+    """The benchmark's budgeted backward: the 17-task ViT-B step through the 64 MiB
+    static array (8 slices) is bitwise the full-workspace backward."""
+    import paper_2608_16188_gb300 as vm
+    cfg = workloads.CONFIGS["vitb_t17"]
+    p = problem_of(cfg)
+    inp = to_dev(workloads.make_inputs(cfg, with_weights=False))
+    inp["w1"], inp["w2"] = workloads.make_weights_fast(cfg, "cuda", seed=5)
+    run = vm.StepRunner(p, inp)
+    run.step()
+    torch.cuda.synchronize()
+    b = run.b
+    ref = [t.clone() for t in (b.dxe, b.dw1, b.dw2)]
+    rows = (torch.arange(b.C, device="cuda")[None, None, :] < b.load[:, :, None])
+    outs = [torch.full_like(t, float("nan")) for t in ref]
+    vm.vmoe_expert_bwd_static_scratch(p, b.xe, b.h, b.a, inp["w1"], inp["w2"], b.dye, b.load, *outs)
+    torch.cuda.synchronize()
+    assert vm.vmoe_device_status() == 0
+    assert torch.equal(outs[0][rows], ref[0][rows])
+    assert torch.equal(outs[1], ref[1]) and torch.equal(outs[2], ref[2])
