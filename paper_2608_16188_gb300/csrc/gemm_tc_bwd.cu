@@ -61,8 +61,8 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
     const int G = p.G();
     const size_t plan_bytes = bwd_plan_bytes(p);
     if (workspace_bytes < bwd_min_workspace(p)) return VMOE_ERR_INVALID;
-    const long long rows = (long long)((workspace_bytes - plan_bytes) / ((size_t)p.f * sizeof(__nv_bfloat16)));
-    const long long cap_units = rows / BW_UNIT;
+    long long rows = (long long)((workspace_bytes - plan_bytes) / ((size_t)p.f * sizeof(__nv_bfloat16)));
+    if (rows > 0x7fffffffLL) rows = 0x7fffffffLL;  // compact row offsets are int32
     std::vector<int32_t> hload(G);
     if (cudaMemcpyAsync(hload.data(), load, sizeof(int32_t) * G, cudaMemcpyDeviceToHost, s) !=
             cudaSuccess ||
@@ -70,12 +70,17 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
         return VMOE_ERR_CUDA;
     std::vector<int64_t> w(G);
     std::vector<double> r(G);
+    long long total_units = 0;
     for (int g = 0; g < G; ++g) {
         const int L = hload[g] < 0 ? 0 : (hload[g] > p.C ? p.C : hload[g]);
         hload[g] = L;
         w[g] = (2LL * L + BW_UNIT - 1) / BW_UNIT;
         r[g] = (double)L;
+        total_units += w[g];
     }
+    // no slice needs more than every group's footprint: that bounds the DP table
+    long long cap_units = rows / BW_UNIT;
+    if (cap_units > total_units) cap_units = total_units;
     std::vector<int32_t> order(G), start(G + 1);
     const int ns = plan_slices(G, w.data(), r.data(), cap_units, 0.0, 0.0, order.data(), start.data());
     if (ns < 0) return ns;
