@@ -156,12 +156,15 @@ route_topk_kernel(Dims p, const TX *__restrict__ x, const float *__restrict__ wr
 // while staging, as packed bf16 pairs along k.
 constexpr int RM_TOK = 64;
 constexpr int RM_THREADS = 128;
-constexpr int RM_KC = 64;
+#ifndef VMOE_ROUTE_KC
+#define VMOE_ROUTE_KC 128
+#endif
+constexpr int RM_KC = VMOE_ROUTE_KC;  // d per staged chunk: 128 halves the chunk chain of 64
 constexpr int RM_XP = RM_KC + 8;  // x row pitch in bf16 (conflict-free fragment loads)
 
 // NB blocks of 8 experts per pass.
 template <int NB>
-__global__ void __launch_bounds__(RM_THREADS)
+__global__ void __launch_bounds__(RM_THREADS, 3)
 route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__restrict__ wr,
                  const float *__restrict__ bias, float *__restrict__ logits,
                  int32_t *__restrict__ out_idx, float *__restrict__ out_gate) {
@@ -275,14 +278,15 @@ int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, co
     constexpr int NP = NB * 8;
     size_t smem = (size_t)RM_TOK * RM_XP * 2 + (size_t)3 * (RM_KC / 2) * (NP + 8) * 4 +
                   (size_t)RM_TOK * (p.E + 1) * 4;
-    static uint64_t attr_done = 0;
+    if (smem > 227 * 1024) return VMOE_ERR_UNSUPPORTED;
+    static int attr_bytes[64];  // per device: the largest size set so far
     int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !(attr_done >> dev & 1ull)) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
+    if (attr_bytes[dev] < (int)smem) {
         if (cudaFuncSetAttribute(route_mma_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 128 * 1024) != cudaSuccess)
+                                 (int)smem) != cudaSuccess)
             return VMOE_ERR_CUDA;
-        attr_done |= 1ull << dev;
+        attr_bytes[dev] = (int)smem;
     }
     dim3 grid((p.N + RM_TOK - 1) / RM_TOK, p.T);
     trace_before(s, "route_topk");
