@@ -6,8 +6,9 @@
 // < T*N*k copies the kept choice w to its slot; warps past that zero the
 // padding rows s >= load of every group, so every element of dst is written
 // exactly once and no memset is needed.  Combine is the gather form of the
-// scatter-add: one warp per token sums its kept choices in the order
-// j = 0..k-1 in fp32 and writes the row once, with no atomics.
+// scatter-add: a warp per token (persistent warps, the next token's routing
+// prefetched) sums its kept choices in the order j = 0..k-1 in fp32 and
+// writes the row once, with no atomics.
 #include "common.cuh"
 
 namespace vmoe {
@@ -96,6 +97,8 @@ dispatch_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ wei
 }
 
 // KMAX >= p.k is a compile-time bound so the gathered rows stay in registers.
+// Persistent warps: warp w takes tokens w, w + W, ... (W warps in the grid)
+// and fetches the next token's routing while the current token's rows load.
 template <typename T, int KMAX>
 __global__ void __launch_bounds__(PM_THREADS)
 combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weight,
@@ -103,56 +106,81 @@ combine_kernel(Dims p, const T *__restrict__ src, const float *__restrict__ weig
                T *__restrict__ dst) {
     pdl_wait();
     constexpr int V = Vec<T>::n;
-    const long long tn = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
-    if (tn >= (long long)p.T * p.N) return;
+    const long long TN = (long long)p.T * p.N;
+    const long long nw = (long long)gridDim.x * PM_WARPS;
+    long long tn = (long long)blockIdx.x * PM_WARPS + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
     const int nvec = p.d / V;
-    const int t = (int)(tn / p.N);
+    int e[KMAX], sl[KMAX];
     float wj[KMAX];
-    const uint4 *rows[KMAX];
-#pragma unroll
-    for (int j = 0; j < KMAX; ++j) {
-        rows[j] = nullptr;
-        wj[j] = 0.0f;
-        if (j < p.k) {
-            const int e = idx[tn * p.k + j], s = slot[tn * p.k + j];
-            wj[j] = weight ? weight[tn * p.k + j] : 1.0f;
-            if (s >= 0)
-                rows[j] = reinterpret_cast<const uint4 *>(
-                    src + (((long long)t * p.E + e) * p.C + s) * p.d);
-        }
-    }
-    uint4 *out = reinterpret_cast<uint4 *>(dst + tn * p.d);
-    // Up to UNR vectors per lane per pass, all k source rows loaded before the
-    // sums, so each warp has k * UNR 16-byte loads in flight.
-    constexpr int UNR = 3;
-    for (int v0 = lane; v0 < nvec; v0 += 32 * UNR) {
-        uint4 buf[KMAX][UNR];
+    auto routing = [&](long long tok, int (&ee)[KMAX], int (&ss)[KMAX], float (&ww)[KMAX]) {
 #pragma unroll
         for (int j = 0; j < KMAX; ++j) {
-            if (rows[j] == nullptr) continue;
+            ee[j] = 0;
+            ss[j] = -1;
+            ww[j] = 0.0f;
+            if (j < p.k && tok < TN) {
+                ee[j] = __ldg(idx + tok * p.k + j);
+                ss[j] = __ldg(slot + tok * p.k + j);
+                ww[j] = weight ? __ldg(weight + tok * p.k + j) : 1.0f;
+            }
+        }
+    };
+    routing(tn, e, sl, wj);
+    for (; tn < TN; tn += nw) {
+        const int t = (int)(tn / p.N);
+        const uint4 *rows[KMAX];
+#pragma unroll
+        for (int j = 0; j < KMAX; ++j)
+            rows[j] = sl[j] >= 0 ? reinterpret_cast<const uint4 *>(
+                                       src + (((long long)t * p.E + e[j]) * p.C + sl[j]) * p.d)
+                                 : nullptr;
+        uint4 *out = reinterpret_cast<uint4 *>(dst + tn * p.d);
+        int e2[KMAX], s2[KMAX];
+        float w2[KMAX];
+        bool next_loaded = false;
+        // Up to UNR vectors per lane per pass, all k source rows loaded before the
+        // sums, so each warp has k * UNR 16-byte loads in flight.
+        constexpr int UNR = 3;
+        for (int v0 = lane; v0 < nvec; v0 += 32 * UNR) {
+            uint4 buf[KMAX][UNR];
+#pragma unroll
+            for (int j = 0; j < KMAX; ++j) {
+                if (rows[j] == nullptr) continue;
+#pragma unroll
+                for (int u = 0; u < UNR; ++u) {
+                    int v = v0 + 32 * u;
+                    if (v < nvec) buf[j][u] = __ldg(rows[j] + v);
+                }
+            }
+            if (!next_loaded) {  // the next token's routing, behind this token's rows
+                routing(tn + nw, e2, s2, w2);
+                next_loaded = true;
+            }
 #pragma unroll
             for (int u = 0; u < UNR; ++u) {
                 int v = v0 + 32 * u;
-                if (v < nvec) buf[j][u] = __ldg(rows[j] + v);
+                if (v >= nvec) continue;
+                float acc[V];
+#pragma unroll
+                for (int q = 0; q < V; ++q) acc[q] = 0.0f;
+#pragma unroll
+                for (int j = 0; j < KMAX; ++j) {  // fixed order j = 0..k-1
+                    if (rows[j] == nullptr) continue;
+                    float f[V];
+                    Vec<T>::load(buf[j][u], f);
+#pragma unroll
+                    for (int q = 0; q < V; ++q) acc[q] = fmaf(wj[j], f[q], acc[q]);
+                }
+                out[v] = Vec<T>::store(acc);
             }
         }
+        if (!next_loaded) routing(tn + nw, e2, s2, w2);
 #pragma unroll
-        for (int u = 0; u < UNR; ++u) {
-            int v = v0 + 32 * u;
-            if (v >= nvec) continue;
-            float acc[V];
-#pragma unroll
-            for (int q = 0; q < V; ++q) acc[q] = 0.0f;
-#pragma unroll
-            for (int j = 0; j < KMAX; ++j) {  // fixed order j = 0..k-1
-                if (rows[j] == nullptr) continue;
-                float f[V];
-                Vec<T>::load(buf[j][u], f);
-#pragma unroll
-                for (int q = 0; q < V; ++q) acc[q] = fmaf(wj[j], f[q], acc[q]);
-            }
-            out[v] = Vec<T>::store(acc);
+        for (int j = 0; j < KMAX; ++j) {
+            e[j] = e2[j];
+            sl[j] = s2[j];
+            wj[j] = w2[j];
         }
     }
 }
@@ -176,20 +204,40 @@ int launch_dispatch(const Dims &p, const void *src, const float *weight, const i
     return st;
 }
 
+// Persistent grid: at most as many CTAs as fit on the GPU at once.
+template <typename T, int KMAX>
+static unsigned combine_grid(long long blocks) {
+    static int per_sm[64];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return (unsigned)blocks;
+    if (per_sm[dev] < 1) {
+        int v = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, combine_kernel<T, KMAX>, PM_THREADS, 0) !=
+                cudaSuccess || v < 1)
+            v = 1;
+        per_sm[dev] = v;
+    }
+    const long long cap = (long long)per_sm[dev] * num_sms();
+    return (unsigned)(blocks < cap ? blocks : cap);
+}
+
 template <typename T>
 static int combine_as(const Dims &p, const void *src, const float *weight, const int32_t *idx,
-                       const int32_t *slot, void *dst, long long blocks, cudaStream_t s) {
+                      const int32_t *slot, void *dst, long long blocks, cudaStream_t s) {
     const T *in = (const T *)src;
     T *out = (T *)dst;
-    const unsigned nb = (unsigned)blocks;
     if (p.k == 1)
-        return launch_kernel(combine_kernel<T, 1>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 1>, dim3(combine_grid<T, 1>(blocks)), dim3(PM_THREADS), 0, s,
+                             p, in, weight, idx, slot, out);
     else if (p.k == 2)
-        return launch_kernel(combine_kernel<T, 2>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 2>, dim3(combine_grid<T, 2>(blocks)), dim3(PM_THREADS), 0, s,
+                             p, in, weight, idx, slot, out);
     else if (p.k <= 4)
-        return launch_kernel(combine_kernel<T, 4>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 4>, dim3(combine_grid<T, 4>(blocks)), dim3(PM_THREADS), 0, s,
+                             p, in, weight, idx, slot, out);
     else
-        return launch_kernel(combine_kernel<T, 8>, dim3(nb), dim3(PM_THREADS), 0, s, p, in, weight, idx, slot, out);
+        return launch_kernel(combine_kernel<T, 8>, dim3(combine_grid<T, 8>(blocks)), dim3(PM_THREADS), 0, s,
+                             p, in, weight, idx, slot, out);
 }
 
 int launch_combine(const Dims &p, const void *src, const float *weight, const int32_t *idx,
