@@ -152,29 +152,38 @@ route_topk_kernel(Dims p, const TX *__restrict__ x, const float *__restrict__ wr
 // partial product is exact in fp32 and the mma.sync m16n8k16 instructions
 // accumulate in fp32, so the logits keep fp32 accuracy at a small fraction of
 // the CUDA-core instruction count.  One CTA = 4 warps x 16 tokens of one task;
-// d is swept in chunks of 64 staged in shared memory; the weight split is done
-// while staging, as packed bf16 pairs along k.
+// d is swept in chunks of RM_KC staged in shared memory.  The weight split is
+// done while staging, two values per conversion, into [part][expert][k]
+// tiles, so that one ldmatrix.x4 gives the B fragments of two 8-expert blocks
+// (and one gives a warp's A fragment).
 constexpr int RM_TOK = 64;
 constexpr int RM_THREADS = 128;
 #ifndef VMOE_ROUTE_KC
 #define VMOE_ROUTE_KC 128
 #endif
 constexpr int RM_KC = VMOE_ROUTE_KC;  // d per staged chunk: 128 halves the chunk chain of 64
-constexpr int RM_XP = RM_KC + 8;  // x row pitch in bf16 (conflict-free fragment loads)
+constexpr int RM_XP = RM_KC + 8;  // row pitch (bf16) of the x and weight tiles: conflict-free ldmatrix
 
-// NB blocks of 8 experts per pass.
+__device__ __forceinline__ void rm_ldsm_x4(uint32_t (&r)[4], const void *smem) {
+    const uint32_t a = (uint32_t)__cvta_generic_to_shared(smem);
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];\n"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+                 : "r"(a));
+}
+
+// NB blocks of 8 experts per pass (NB even).
 template <int NB>
 __global__ void __launch_bounds__(RM_THREADS, 3)
 route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__restrict__ wr,
                  const float *__restrict__ bias, float *__restrict__ logits,
                  int32_t *__restrict__ out_idx, float *__restrict__ out_gate) {
+    static_assert(NB % 2 == 0, "B fragments are loaded two expert blocks at a time");
     pdl_wait();
     constexpr int NP = NB * 8;
-    constexpr int WP = NP + 8;  // packed-pair row pitch in 32-bit words
     extern __shared__ __align__(16) uint8_t rm_smem[];
-    __nv_bfloat16 *xs = reinterpret_cast<__nv_bfloat16 *>(rm_smem);            // [64][RM_XP]
-    uint32_t *wp = reinterpret_cast<uint32_t *>(xs + RM_TOK * RM_XP);           // [3][RM_KC/2][WP]
-    float *lg = reinterpret_cast<float *>(wp + 3 * (RM_KC / 2) * WP);           // [64][E+1]
+    __nv_bfloat16 *xs = reinterpret_cast<__nv_bfloat16 *>(rm_smem);  // [64][RM_XP]
+    __nv_bfloat16 *ws = xs + RM_TOK * RM_XP;                         // [3][NP][RM_XP]
+    float *lg = reinterpret_cast<float *>(ws + 3 * NP * RM_XP);      // [64][E+1]
     const int t = blockIdx.y, n0 = blockIdx.x * RM_TOK;
     const int E = p.E, d = p.d, N = p.N;
     const int ldl = E + 1;
@@ -183,13 +192,14 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
     const int ntok = min(RM_TOK, N - n0);
     const __nv_bfloat16 *xt = x + ((long long)t * N + n0) * d;
     const float *wt = wr + (long long)t * d * E;
-    // Per thread and chunk: XV x vectors (16 B each) and WV weight pairs.  The
-    // next chunk's values are loaded into registers before the current chunk's
-    // MMAs run, so global latency overlaps the tensor-core work.
+    // Per thread and chunk: XV x vectors (16 B each) and WI weight items, an
+    // item being 8 consecutive k of one expert.  The next chunk's values are
+    // loaded into registers before the current chunk's MMAs run, so global
+    // latency overlaps the tensor-core work.
     constexpr int XV = RM_TOK * (RM_KC / 8) / RM_THREADS;
-    constexpr int WV = (RM_KC / 2) * NP / RM_THREADS;
+    constexpr int WI = (RM_KC / 8) * NP / RM_THREADS;
     uint4 xv[XV];
-    float wv[WV][2];
+    float wv[WI][8];
     auto load_chunk = [&](int e0, int k0) {
 #pragma unroll
         for (int q = 0; q < XV; ++q) {
@@ -200,11 +210,12 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
                 xv[q] = __ldg(reinterpret_cast<const uint4 *>(xt + (long long)r * d + k0 + c));
         }
 #pragma unroll
-        for (int q = 0; q < WV; ++q) {
+        for (int q = 0; q < WI; ++q) {  // consecutive threads: consecutive experts (coalesced)
             const int i = tid + q * RM_THREADS;
-            const int kp = i / NP, n = i % NP, e = e0 + n, dd = k0 + 2 * kp;
-            wv[q][0] = (e < E && dd < d) ? __ldg(wt + (long long)dd * E + e) : 0.0f;
-            wv[q][1] = (e < E && dd + 1 < d) ? __ldg(wt + (long long)(dd + 1) * E + e) : 0.0f;
+            const int n = i % NP, e = e0 + n, kk = k0 + (i / NP) * 8;
+#pragma unroll
+            for (int r = 0; r < 8; ++r)
+                wv[q][r] = (e < E && kk + r < d) ? __ldg(wt + (long long)(kk + r) * E + e) : 0.0f;
         }
     };
     auto stage_chunk = [&]() {
@@ -215,17 +226,31 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
             *reinterpret_cast<uint4 *>(xs + r * RM_XP + c) = xv[q];
         }
 #pragma unroll
-        for (int q = 0; q < WV; ++q) {
+        for (int q = 0; q < WI; ++q) {
             const int i = tid + q * RM_THREADS;
-            const int kp = i / NP, n = i % NP;
-            __nv_bfloat16 h0, m0, l0, h1, m1, l1;
-            split3(wv[q][0], h0, m0, l0);
-            split3(wv[q][1], h1, m1, l1);
-            wp[(0 * (RM_KC / 2) + kp) * WP + n] = pack2(h0, h1);
-            wp[(1 * (RM_KC / 2) + kp) * WP + n] = pack2(m0, m1);
-            wp[(2 * (RM_KC / 2) + kp) * WP + n] = pack2(l0, l1);
+            const int n = i % NP, c = (i / NP) * 8;
+            uint32_t hi[4], mid[4], lo[4];
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {  // split3 of a k pair, both values per conversion
+                const __nv_bfloat162 h = __floats2bfloat162_rn(wv[q][2 * j], wv[q][2 * j + 1]);
+                const float2 hf = __bfloat1622float2(h);
+                const float r0 = wv[q][2 * j] - hf.x, r1 = wv[q][2 * j + 1] - hf.y;
+                const __nv_bfloat162 m = __floats2bfloat162_rn(r0, r1);
+                const float2 mf = __bfloat1622float2(m);
+                const __nv_bfloat162 l = __floats2bfloat162_rn(r0 - mf.x, r1 - mf.y);
+                hi[j] = *reinterpret_cast<const uint32_t *>(&h);
+                mid[j] = *reinterpret_cast<const uint32_t *>(&m);
+                lo[j] = *reinterpret_cast<const uint32_t *>(&l);
+            }
+            *reinterpret_cast<uint4 *>(ws + (0 * NP + n) * RM_XP + c) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
+            *reinterpret_cast<uint4 *>(ws + (1 * NP + n) * RM_XP + c) = make_uint4(mid[0], mid[1], mid[2], mid[3]);
+            *reinterpret_cast<uint4 *>(ws + (2 * NP + n) * RM_XP + c) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
     };
+    // ldmatrix row addresses: A, rows warp*16 + (lane & 15), k offset 8 (lane >> 4);
+    // B, expert (lane & 7) + 8 (lane >> 4) of a block pair, k offset 8 ((lane >> 3) & 1)
+    const __nv_bfloat16 *xa = xs + (warp * 16 + (lane & 15)) * RM_XP + (lane >> 4) * 8;
+    const __nv_bfloat16 *wb = ws + ((lane & 7) + (lane >> 4) * 8) * RM_XP + ((lane >> 3) & 1) * 8;
     for (int e0 = 0; e0 < E; e0 += NP) {
         float acc[NB][4];
 #pragma unroll
@@ -240,18 +265,18 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
             if (k0 + RM_KC < d) load_chunk(e0, k0 + RM_KC);
 #pragma unroll
             for (int ks = 0; ks < RM_KC; ks += 16) {
-                const __nv_bfloat16 *xr = xs + (warp * 16 + g) * RM_XP + ks + 2 * tq;
-                const uint32_t a0 = *reinterpret_cast<const uint32_t *>(xr);
-                const uint32_t a1 = *reinterpret_cast<const uint32_t *>(xr + 8 * RM_XP);
-                const uint32_t a2 = *reinterpret_cast<const uint32_t *>(xr + 8);
-                const uint32_t a3 = *reinterpret_cast<const uint32_t *>(xr + 8 * RM_XP + 8);
+                uint32_t a[4];
+                rm_ldsm_x4(a, xa + ks);
 #pragma unroll
-                for (int nb = 0; nb < NB; ++nb) {
+                for (int np = 0; np < NB / 2; ++np) {
+                    uint32_t b[3][4];  // [part][b0, b1 of block 2np; b0, b1 of block 2np+1]
 #pragma unroll
-                    for (int sp = 2; sp >= 0; --sp) {  // smallest part first
-                        const uint32_t *wrow = wp + (sp * (RM_KC / 2) + ks / 2 + tq) * WP + nb * 8 + g;
-                        mma_bf16_16816(acc[nb], a0, a1, a2, a3, wrow[0], wrow[4 * WP]);
-                    }
+                    for (int sp = 0; sp < 3; ++sp) rm_ldsm_x4(b[sp], wb + (sp * NP + np * 16) * RM_XP + ks);
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+#pragma unroll
+                        for (int sp = 2; sp >= 0; --sp)  // smallest part first
+                            mma_bf16_16816(acc[2 * np + h], a[0], a[1], a[2], a[3], b[sp][2 * h], b[sp][2 * h + 1]);
                 }
             }
         }
@@ -276,8 +301,7 @@ template <int NB>
 int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, const float *bias,
                       float *logits, int32_t *idx, float *gate, cudaStream_t s) {
     constexpr int NP = NB * 8;
-    size_t smem = (size_t)RM_TOK * RM_XP * 2 + (size_t)3 * (RM_KC / 2) * (NP + 8) * 4 +
-                  (size_t)RM_TOK * (p.E + 1) * 4;
+    size_t smem = (size_t)RM_TOK * RM_XP * 2 + (size_t)3 * NP * RM_XP * 2 + (size_t)RM_TOK * (p.E + 1) * 4;
     if (smem > 227 * 1024) return VMOE_ERR_UNSUPPORTED;
     static int attr_bytes[64];  // per device: the largest size set so far
     int dev = 0;
