@@ -320,15 +320,15 @@ int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, co
     return st;
 }
 
-constexpr int CS_THREADS = 256;
-constexpr int CS_WARPS = CS_THREADS / 32;
-
 // SMEM_IDX: the task's idx array and the temporary ranks live in shared memory
 // (read and written with coalesced accesses); otherwise they stay in global memory.
-template <bool SMEM_IDX>
+// CS_THREADS: 1024 (32 warps, 4 rounds of 32 assignments per warp at N k = 3152)
+// while the per-warp expert counters stay small (E <= 128), else 256.
+template <bool SMEM_IDX, int CS_THREADS>
 __global__ void __launch_bounds__(CS_THREADS)
 capacity_scan_kernel(Dims p, const int32_t *__restrict__ idx, int32_t *__restrict__ slot,
                      int32_t *__restrict__ load) {
+    constexpr int CS_WARPS = CS_THREADS / 32;
     pdl_wait();
     extern __shared__ int cs_smem[];
     int *cnt = cs_smem;  // [CS_WARPS][E]
@@ -418,6 +418,27 @@ int launch_topk(const Dims &p, const TX *x, const float *wr, const float *bias, 
     return launch_result();
 }
 
+template <int CS_THREADS>
+int launch_scan(const Dims &p, const int32_t *idx, int32_t *slot, int32_t *load, cudaStream_t s) {
+    const size_t total = (size_t)p.N * p.k;
+    const size_t smem_small = sizeof(int) * (size_t)(CS_THREADS / 32) * p.E;
+    const size_t smem_big = smem_small + sizeof(int) * 2 * total;
+    if (smem_big <= 96 * 1024) {
+        static uint64_t attr_done = 0;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        if (dev < 64 && !(attr_done >> dev & 1ull)) {
+            cudaFuncSetAttribute(capacity_scan_kernel<true, CS_THREADS>,
+                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
+            attr_done |= 1ull << dev;
+        }
+        return launch_kernel(capacity_scan_kernel<true, CS_THREADS>, dim3(p.T), dim3(CS_THREADS), smem_big,
+                             s, p, idx, slot, load);
+    }
+    return launch_kernel(capacity_scan_kernel<false, CS_THREADS>, dim3(p.T), dim3(CS_THREADS), smem_small,
+                         s, p, idx, slot, load);
+}
+
 }  // namespace
 
 int launch_route(const Dims &p, const void *x, const float *w_router, const float *bias,
@@ -436,25 +457,8 @@ int launch_route(const Dims &p, const void *x, const float *w_router, const floa
                        : launch_topk<float, 64>(p, xf, w_router, bias, logits, idx, gate, s);
     }
     if (st != VMOE_OK) return st;
-    const size_t total = (size_t)p.N * p.k;
-    const size_t smem_small = sizeof(int) * (size_t)CS_WARPS * p.E;
-    const size_t smem_big = smem_small + sizeof(int) * 2 * total;
     trace_before(s, "capacity_scan");
-    if (smem_big <= 96 * 1024) {
-        static uint64_t attr_done = 0;
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev < 64 && !(attr_done >> dev & 1ull)) {
-            cudaFuncSetAttribute(capacity_scan_kernel<true>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
-            attr_done |= 1ull << dev;
-        }
-        st = launch_kernel(capacity_scan_kernel<true>, dim3(p.T), dim3(CS_THREADS), smem_big, s, p,
-                           idx, slot, load);
-    } else {
-        st = launch_kernel(capacity_scan_kernel<false>, dim3(p.T), dim3(CS_THREADS), smem_small, s,
-                           p, idx, slot, load);
-    }
+    st = p.E <= 128 ? launch_scan<1024>(p, idx, slot, load, s) : launch_scan<256>(p, idx, slot, load, s);
     trace_after(s);
     return st;
 }
