@@ -106,6 +106,22 @@ struct Args {
     int compact;               // CMP_* bits
 };
 enum { CMP_A = 1, CMP_B = 2, CMP_D = 4 };
+
+// Partial-box tensor maps: a group's padding rows [load, C) are not read.
+// Row mode: a[0..2] = the A operand with 64-, 32- and 16-row boxes; a tile
+// whose valid rows end inside it loads rows [0, 16 ceil(rows / 16)) as at most
+// three boxes instead of one 128-row box.
+// Weight gradients, resident-B kernel: a[i], b[i] = the A and B operands with
+// boxes of 16 (i + 1) K rows, for a group's last k-block when its valid rows
+// end inside it.  Such a box lands chunk-major with a chunk stride of
+// (rows x 128) bytes, which the k-block's MMA descriptors take as their
+// leading byte offset.
+struct TailMaps {
+    CUtensorMap a[3], b[3];
+};
+// Rows loaded for a k-block with `rem` valid K rows (>= 1): all BK, or rem
+// rounded up to 16.
+__host__ __device__ __forceinline__ int tail_rows(int rem) { return rem >= 64 ? 64 : ((rem + 15) & ~15); }
 __device__ __forceinline__ int real_group(const Args &a, int i) { return a.glist ? __ldg(a.glist + i) : i; }
 
 // ---------------------------------------------------------------------------
@@ -272,6 +288,10 @@ __device__ __forceinline__ uint64_t operand_desc(uint32_t tile, int kk, bool mn_
     return mn_major ? sdesc_sw128(tile + kk * 2048, 8192, 1024)
                     : sdesc_sw128(tile + kk * 32, 16, 1024);
 }
+// MN-major k-block of `rows` K rows: its MN chunks are rows x 128 bytes apart.
+__device__ __forceinline__ uint64_t operand_desc_mn(uint32_t tile, int kk, int rows) {
+    return sdesc_sw128(tile + kk * 2048, (uint32_t)rows * 128u, 1024);
+}
 
 // Instruction descriptor of tcgen05.mma kind::f16: D fp32 (bits 4-5 = 1),
 // A and B bf16 (bits 7-9, 10-12 = 1), A / B MN-major (bits 15 / 16),
@@ -329,7 +349,7 @@ template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
 __global__ void __launch_bounds__(THREADS, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmD, const __grid_constant__ CUtensorMap tmD2,
-                    Args args) {
+                    const __grid_constant__ TailMaps tmAt, Args args) {
     using S = Shape<BN, MODE, EPI>;
     constexpr int STAGES = S::STAGES;
     constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
@@ -367,6 +387,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         fence_proxy_async();
         prefetch_map(&tmA);
         prefetch_map(&tmB);
+        if (MODE == MODE_ROW)
+            for (int i = 0; i < 3; ++i) prefetch_map(&tmAt.a[i]);
     }
     if (warp == 0) {
         tmem_alloc(smem_u32(misc), S::TMEM_COLS);
@@ -447,11 +469,28 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                     const uint32_t sb = sa + S::A_BYTES;
                     const uint32_t fb = bar_full(stage);
                     if (MODE == MODE_ROW) {
-                        mbar_expect_tx(fb, S::STAGE_BYTES);
-                        if (args.compact & CMP_A)
-                            tma_load_3d(sa, &tmA, fb, kb * BK, t.crow + t.m_blk * BM, 0);
-                        else
-                            tma_load_3d(sa, &tmA, fb, kb * BK, t.m_blk * BM, t.gr);
+                        // A rows [0, rn): the tile's valid rows rounded up to 16.  The
+                        // slot's rows past rn keep stale data, which only reaches
+                        // output rows past rows_valid -- never stored.
+                        const int rem_rows = t.rows_valid - t.m_blk * BM;
+                        const int rn = rem_rows >= BM ? BM : ((rem_rows + 15) & ~15);
+                        const bool cmpa = (args.compact & CMP_A) != 0;
+                        const int r0 = (cmpa ? t.crow : 0) + t.m_blk * BM, gz = cmpa ? 0 : t.gr;
+                        mbar_expect_tx(fb, (uint32_t)rn * (BK * 2) + S::B_BYTES);
+                        if (rn == BM) {
+                            tma_load_3d(sa, &tmA, fb, kb * BK, r0, gz);
+                        } else {
+                            int off = 0;
+                            if (rn & 64) {
+                                tma_load_3d(sa, &tmAt.a[0], fb, kb * BK, r0, gz);
+                                off = 64;
+                            }
+                            if (rn & 32) {
+                                tma_load_3d(sa + off * (BK * 2), &tmAt.a[1], fb, kb * BK, r0 + off, gz);
+                                off += 32;
+                            }
+                            if (rn & 16) tma_load_3d(sa + off * (BK * 2), &tmAt.a[2], fb, kb * BK, r0 + off, gz);
+                        }
                         if (B_MN) {  // one 4-D box: BN/64 column chunks of 64 rows
                             tma_load_4d(sb, &tmB, fb, 0, kb * BK, t.n_blk * (BN / 64), t.gr);
                         } else {
@@ -461,6 +500,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                         // Weight gradients: K = the group's rows.  With ksplit the second
                         // half of the k-blocks pairs the same A rows with B's residual
                         // rows, which start at row C of the group.
+                        // (Tail-sized boxes for the last k-block, as in the resident-B
+                        // kernel, made this streaming kernel slower: full boxes here.)
                         mbar_expect_tx(fb, S::STAGE_BYTES);
                         const int hi = (kb >= t.khalf) ? 1 : 0;
                         const int ka = (kb - hi * t.khalf) * BK;
@@ -959,7 +1000,8 @@ struct BStatShape {
 template <int BN, bool KSPLIT, int B_BUFS>
 __global__ void __launch_bounds__(THREADS, 1)
 wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                   const __grid_constant__ CUtensorMap tmD, Args args) {
+                   const __grid_constant__ CUtensorMap tmD, const __grid_constant__ TailMaps tmT,
+                   Args args) {
     using S = BStatShape<BN, KSPLIT, B_BUFS>;
     constexpr uint32_t IDESC = idesc_bf16(BM, BN, true, true);
     extern __shared__ uint8_t smem_raw[];
@@ -998,6 +1040,10 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         prefetch_map(&tmA);
         prefetch_map(&tmB);
         prefetch_map(&tmD);
+        for (int i = 0; i < 3; ++i) {
+            prefetch_map(&tmT.a[i]);
+            prefetch_map(&tmT.b[i]);
+        }
     }
     if (warp == 0) {
         tmem_alloc(smem_u32(misc), S::TMEM_COLS);
@@ -1043,13 +1089,17 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                                 args.status))
                     break;
                 const uint32_t bdst = smem_u32(b_res) + bb * S::B_BYTES;
-                mbar_expect_tx(bar_bfull(bb), (uint32_t)(nkb * (KSPLIT ? 2 : 1)) * S::B_KB);
+                // the last k-block loads R = tail_rows(rem) rows (chunk stride R x 128)
+                const int Rl = tail_rows(L - (nkb - 1) * BK);
+                const uint32_t bbytes = (uint32_t)((nkb - 1) * BK + Rl) * (BN / 64) * 128u;
+                mbar_expect_tx(bar_bfull(bb), (KSPLIT ? 2u : 1u) * bbytes);
                 const bool cmpb = (args.compact & CMP_B) != 0;  // B rows from crow, residual after L
                 for (int kb = 0; kb < nkb; ++kb) {
-                    tma_load_4d(bdst + kb * S::B_KB, &tmB, bar_bfull(bb), 0,
+                    const CUtensorMap *mB = kb == nkb - 1 && Rl < BK ? &tmT.b[Rl / 16 - 1] : &tmB;
+                    tma_load_4d(bdst + kb * S::B_KB, mB, bar_bfull(bb), 0,
                                 (cmpb ? crow : 0) + kb * BK, n_blk * (BN / 64), cmpb ? 0 : g);
                     if (KSPLIT)
-                        tma_load_4d(bdst + (2 + kb) * S::B_KB, &tmB, bar_bfull(bb), 0,
+                        tma_load_4d(bdst + (2 + kb) * S::B_KB, mB, bar_bfull(bb), 0,
                                     (cmpb ? crow + L : args.C) + kb * BK, n_blk * (BN / 64),
                                     cmpb ? 0 : g);
                 }
@@ -1062,9 +1112,10 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                         ok = false;
                         break;
                     }
-                    mbar_expect_tx(bar_afull(ab), (uint32_t)nkb * S::A_KB);
+                    mbar_expect_tx(bar_afull(ab), (uint32_t)((nkb - 1) * BK + Rl) * (BM / 64) * 128u);
                     for (int kb = 0; kb < nkb; ++kb)
-                        tma_load_4d(smem_u32(a_ring) + ab * S::A_BUF + kb * S::A_KB, &tmA,
+                        tma_load_4d(smem_u32(a_ring) + ab * S::A_BUF + kb * S::A_KB,
+                                    kb == nkb - 1 && Rl < BK ? &tmT.a[Rl / 16 - 1] : &tmA,
                                     bar_afull(ab), 0, kb * BK, m * (BM / 64), g);
                     ++a_issued[ab];
                 }
@@ -1089,14 +1140,15 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
         int ub = 0;
         int ia = 0, it = 0;
         bool ok = true;
-        // rows [z0, z1) of every 64-wide chunk of a k-block tile are zeroed
+        // rows [z0, z1) of every 64-wide chunk of the last k-block tile, whose
+        // chunks are z1 x 128 bytes apart (it holds z1 = tail_rows rows), are zeroed
         auto zero_rows = [&](uint8_t *tile, int chunks, int z0, int z1) {
             const int rows = z1 - z0;
             const int units = chunks * rows * 8;
             for (int i = lane; i < units; i += 32) {
                 const int c = i / (rows * 8);
                 const int w = i - c * rows * 8;
-                *reinterpret_cast<uint4 *>(tile + c * 8192 + (z0 + (w >> 3)) * 128 + (w & 7) * 16) =
+                *reinterpret_cast<uint4 *>(tile + c * (z1 * 128) + (z0 + (w >> 3)) * 128 + (w & 7) * 16) =
                     make_uint4(0, 0, 0, 0);
             }
         };
@@ -1152,8 +1204,8 @@ wgrad_bstat_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constan
                             const int nk = kb == nkb - 1 ? nk_last : BK / 16;
                             const uint32_t at = a0 + kb * S::A_KB;
                             const uint32_t bt = b0 + (part * 2 + kb) * S::B_KB;
-                            for (int kk = 0; kk < nk; ++kk)
-                                mma_bf16(dtmem, operand_desc(at, kk, true), operand_desc(bt, kk, true),
+                            for (int kk = 0; kk < nk; ++kk)  // k-block of 16 nk rows (the last one: tail_rows)
+                                mma_bf16(dtmem, operand_desc_mn(at, kk, nk * 16), operand_desc_mn(bt, kk, nk * 16),
                                          IDESC, (part | kb | kk) != 0 ? 1u : 0u);
                         }
                     mma_commit(bar_aempty(ab));
@@ -1271,8 +1323,8 @@ bool make_map_chunked(CUtensorMap *map, const void *base, uint64_t mn, uint64_t 
 
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
 int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
-           const CUtensorMap &md2, const Args &a, long long max_tiles, cudaStream_t s,
-           const char *name) {
+           const CUtensorMap &md2, const TailMaps &mat, const Args &a, long long max_tiles,
+           cudaStream_t s, const char *name) {
     using S = Shape<BN, MODE, EPI>;
     auto kern = grouped_gemm_kernel<BN, MODE, A_MN, B_MN, EPI>;
     static uint64_t attr_done = 0;  // one bit per device
@@ -1288,14 +1340,14 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
     const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(THREADS), S::SMEM_BYTES, s, ma, mb,
-                                 md, md2, a);
+                                 md, md2, mat, a);
     trace_after(s);
     return st;
 }
 
 template <int BN, bool KSPLIT, int B_BUFS>
-int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md, const Args &a,
-                 long long units, cudaStream_t s, const char *name) {
+int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md, const TailMaps &mt,
+                 const Args &a, long long units, cudaStream_t s, const char *name) {
     using S = BStatShape<BN, KSPLIT, B_BUFS>;
     auto kern = wgrad_bstat_kernel<BN, KSPLIT, B_BUFS>;
     static uint64_t attr_done = 0;  // one bit per device
@@ -1311,7 +1363,7 @@ int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap
     long long grid = units < num_sms() ? units : num_sms();
     trace_before(s, name);
     const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(THREADS), S::SMEM_BYTES, s, ma, mb,
-                                 md, a);
+                                 md, mt, a);
     trace_after(s);
     return st;
 }
@@ -1351,9 +1403,14 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
     CUtensorMap ma, mb;
-    const bool okA = (sl.compact & CMP_A) ? make_map(&ma, act, K, (uint64_t)sl.rows, 1, 128)
-                                          : make_map(&ma, act, K, C, G, 128, (uint64_t)sAct);
-    if (!okA) return VMOE_ERR_CUDA;
+    TailMaps mat;
+    const bool cmpa = (sl.compact & CMP_A) != 0;
+    auto amap = [&](CUtensorMap *m, uint32_t box) {
+        return cmpa ? make_map(m, act, K, (uint64_t)sl.rows, 1, box)
+                    : make_map(m, act, K, C, G, box, (uint64_t)sAct);
+    };
+    if (!amap(&ma, 128) || !amap(&mat.a[0], 64) || !amap(&mat.a[1], 32) || !amap(&mat.a[2], 16))
+        return VMOE_ERR_CUDA;
     bool okb = B_MN ? make_map_chunked(&mb, w, N, K, G, 64, BN / 64) : make_map(&mb, w, K, N, G, BN);
     if (!okb) return VMOE_ERR_CUDA;
     Args a = base_args(p, load);
@@ -1379,8 +1436,8 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
         if (!make_map(&md, D, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
         if (D2 && !make_map(&md2, D2, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
     }
-    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, a, max_tiles, s, name)
-                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, a, max_tiles, s, name);
+    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name)
+                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name);
 }
 
 // Weight-gradient GEMM: D[g][M][N] = act1[g][C][M]^T * act2[g][C][N], summed
@@ -1398,6 +1455,15 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
     const uint64_t b_rows = cmpb ? (uint64_t)sl.rows : (uint64_t)(ksplit ? 2 * C : C);
     const uint64_t b_outer = cmpb ? 1 : (uint64_t)G;
     CUtensorMap ma, mb, md;
+    TailMaps mt;  // the last k-block's boxes of 16, 32 and 48 K rows
+    // b_chunks: the B tile's 64-column chunks (the kernel's BN / 64)
+    auto tail_maps = [&](int b_chunks) {
+        for (int i = 0; i < 3; ++i)
+            if (!make_map_chunked(&mt.a[i], act1, M, C, G, 16 * (i + 1), BM / 64) ||
+                !make_map_chunked(&mt.b[i], act2, N, b_rows, b_outer, 16 * (i + 1), b_chunks))
+                return false;
+        return true;
+    };
     if (!make_map_chunked(&ma, act1, M, C, G, 64, BM / 64)) return VMOE_ERR_CUDA;
     if (!make_map_chunked(&mb, act2, N, b_rows, b_outer, 64, BN / 64)) return VMOE_ERR_CUDA;
     if (!make_map(&md, D, N, M, G, 32)) return VMOE_ERR_CUDA;  // 64 x 32 store boxes
@@ -1420,14 +1486,16 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
         using SB = BStatShape<BSTAT_BN, true, BSTAT_BUFS>;
         CUtensorMap mbs;
         if (!make_map_chunked(&mbs, act2, N, b_rows, b_outer, 64, BSTAT_BN / 64)) return VMOE_ERR_CUDA;
+        if (!tail_maps(BSTAT_BN / 64)) return VMOE_ERR_CUDA;
         a.tiles_n = N / BSTAT_BN;
         const int nch = (a.tiles_m + SB::MCH - 1) / SB::MCH;
         const long long units = (long long)a.G * a.tiles_n * nch;
-        return launch_bstat<BSTAT_BN, true, BSTAT_BUFS>(ma, mbs, md, a, units, s, name);
+        return launch_bstat<BSTAT_BN, true, BSTAT_BUFS>(ma, mbs, md, mt, a, units, s, name);
     }
     long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
-    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name)
-                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, a, max_tiles, s, name);
+    const TailMaps unused{};  // the streaming kernel loads full k-blocks
+    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, unused, a, max_tiles, s, name)
+                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, unused, a, max_tiles, s, name);
 }
 
 }  // namespace tc
