@@ -137,6 +137,8 @@ int vmoe_dispatch(const vmoe_problem *p, const void *src, const float *weight,
  *   H = Xe W1, A = GELU(H), Ye = A W2, per group g for its rows s < load[g].
  *   xe [T,E,C,d], w1 [T,E,d,f], w2 [T,E,f,d], load [T,E] int32
  *   h, a [T,E,C,f] out, ye [T,E,C,d] out -- rows s >= load[g] are not written.
+ * Rows s >= load[g] of xe are padding: their contents (NaN included) reach no
+ * output.  load[g] is clamped to [0, C].
  * bf16: fp32 accumulation; A is GELU of the fp32 accumulator, H and A are
  * stored rounded to bf16. */
 int vmoe_expert_fwd(const vmoe_problem *p, const void *xe, const void *w1, const void *w2,
@@ -162,6 +164,8 @@ size_t vmoe_expert_bwd_min_workspace_size(const vmoe_problem *p);
  *   (= vmoe_dispatch(dY, gate)), load [T,E]
  *   dxe [T,E,C,d] out (rows >= load not written), dw1 [T,E,d,f] out, dw2 [T,E,f,d] out
  *   (every element written; zero for a group with load 0)
+ *   Rows s >= load[g] of xe, h, a and dye are padding: their contents (NaN
+ *   included) reach no output.
  *   workspace: caller-owned device scratch, 16-byte aligned, its contents
  *   clobbered.  With vmoe_expert_bwd_workspace_size(p) bytes or more, dH of
  *   every group fits and the call is asynchronous.  bf16 problems also accept

@@ -26,6 +26,7 @@ struct SimtArgs {
     int lda, ldb, ldd;
     int M, N, K;  // fixed sizes (M ignored in row mode, K ignored in wgrad mode)
     const int32_t *load;
+    int C;         // capacity: load[g] is clamped to [0, C], as in the tensor-core path
     int row_mode;  // 1: M = load[g]; 0: K = load[g]
     int gelu_tanh;
 };
@@ -37,7 +38,8 @@ __global__ void __launch_bounds__(256) simt_gemm_kernel(SimtArgs a) {
     __shared__ float As[ST_BK][ST_BM + 4];
     __shared__ float Bs[ST_BK][ST_BN + 4];
     const int g = blockIdx.z;
-    const int Lg = a.load[g];
+    int Lg = a.load[g];
+    Lg = Lg < 0 ? 0 : (Lg > a.C ? a.C : Lg);
     const int M = a.row_mode ? Lg : a.M;
     const int K = a.row_mode ? a.K : Lg;
     const int m0 = blockIdx.y * ST_BM, n0 = blockIdx.x * ST_BN;
@@ -113,6 +115,7 @@ int run(const SimtArgs &a, int G, int mmax, cudaStream_t s, const char *name) {
 
 SimtArgs base(const Dims &p) {
     SimtArgs a = {};
+    a.C = p.C;
     a.gelu_tanh = (p.flags & VMOE_GELU_TANH) != 0;
     return a;
 }
