@@ -17,13 +17,14 @@
 // has k non-zeros, so the update is k scaled columns of W_r, not an E-term
 // contraction.
 //
-// Kernel 2 (router_dw), bf16 problems: dW_r = x^T dlogit on the tensor cores.
-// x is exact in bf16; dlogit (fp32) is split into three bf16 parts while it is
-// staged, so every partial product is exact in fp32 and mma.sync accumulates
-// in fp32.  The token (reduction) dimension is split over the 4 CTAs of a
-// thread-block cluster and the partial tiles are summed through distributed
-// shared memory in rank order, so the result is deterministic.  fp32 problems
-// use a CUDA-core tile kernel instead.  No atomics anywhere.
+// Kernel 2 (router_dw), bf16 problems: dW_r = x^T dlogit on the tensor cores,
+// tcgen05 for E = 32 or 64 and d a multiple of 128 (router_dw_tc.cu), else the
+// mma.sync kernel below.  x is exact in bf16; dlogit (fp32) is split into three
+// bf16 parts while it is staged, so every partial product is exact in fp32 and
+// the MMAs accumulate in fp32.  The token (reduction) dimension is split over
+// the CTAs of a thread-block cluster and the partial tiles are summed through
+// distributed shared memory in rank order, so the result is deterministic.
+// fp32 problems use a CUDA-core tile kernel instead.  No atomics anywhere.
 #include <cooperative_groups.h>
 #include <math.h>
 
@@ -34,6 +35,10 @@
 namespace cg = cooperative_groups;
 
 namespace vmoe {
+
+int launch_router_dw_tc(const Dims &p, const __nv_bfloat16 *x, const float *dl, float *dw, float *dbias,
+                        cudaStream_t s);  // router_dw_tc.cu
+
 namespace {
 
 // ---------------------------------------------------------------------------
@@ -901,6 +906,11 @@ int run(const Dims &p, const void *x, const float *wr, const float *logits, cons
     trace_after(s);
     if (st != VMOE_OK) return st;
     trace_before(s, "router_dw");
+    if (p.bf16 && (st = launch_router_dw_tc(p, (const __nv_bfloat16 *)x, dlogits, dw, dbias, s)) !=
+                      VMOE_ERR_UNSUPPORTED) {
+        trace_after(s);
+        return st;
+    }
     if (p.bf16) {
         dim3 grid(DW_SPLIT, (p.d + DW_BD - 1) / DW_BD, p.T * ((p.E + DW_BE - 1) / DW_BE));
         router_dw_mma_kernel<<<grid, DW_THREADS, 0, s>>>(p, (const __nv_bfloat16 *)x, dlogits, dw,
