@@ -16,6 +16,7 @@
 #include <stdint.h>
 
 #include <algorithm>
+#include <memory>
 #include <numeric>
 #include <vector>
 
@@ -45,23 +46,32 @@ int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t ca
     for (int i : sjf) (weight[i] == 0 ? zero : remaining).push_back(i);
 
     std::vector<std::vector<int>> slices;
-    std::vector<double> dp(cap + 1);
-    std::vector<uint8_t> take;
+    // Two DP rows, row a-1 (cur) -> row a (nxt): every entry of row a depends on
+    // row a-1 only, so the update is branch-free and vectorises; the decision
+    // table gets every entry written, so it needs no clearing.
+    std::vector<double> cur(cap + 1), nxt(cap + 1);
+    std::unique_ptr<uint8_t[]> take(new uint8_t[(size_t)n * (cap + 1)]);
     while (!remaining.empty()) {
         const int m = (int)remaining.size();
-        std::fill(dp.begin(), dp.end(), 0.0);
-        take.assign((size_t)m * (cap + 1), 0);
+        std::fill(cur.begin(), cur.end(), 0.0);
         for (int a = 0; a < m; ++a) {
             const int i = remaining[a];
             const int wi = (int)weight[i];
-            uint8_t *t = take.data() + (size_t)a * (cap + 1);
-            for (int j = cap; j >= wi; --j) {  // descending: dp[j - wi] is still row a-1
-                const double cand = dp[j - wi] + v[i];
-                if (cand > dp[j]) {
-                    dp[j] = cand;
-                    t[j] = 1;
-                }
+            const double vi = v[i];
+            uint8_t *__restrict__ t = take.get() + (size_t)a * (cap + 1);
+            const double *__restrict__ o = cur.data();
+            double *__restrict__ nw = nxt.data();
+            for (int j = 0; j < wi; ++j) {
+                nw[j] = o[j];
+                t[j] = 0;
             }
+            for (int j = wi; j <= cap; ++j) {  // taken only when strictly better
+                const double cand = o[j - wi] + vi;
+                const bool tk = cand > o[j];
+                nw[j] = tk ? cand : o[j];
+                t[j] = tk;
+            }
+            cur.swap(nxt);
         }
         std::vector<uint8_t> chosen(n, 0);
         int nchosen = 0;
