@@ -51,16 +51,16 @@ constexpr unsigned long long TIMEOUT_NS = 4000000000ull;
 enum { MODE_ROW = 0, MODE_WGRAD = 1 };
 enum { EPI_STORE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
 
-// Epilogue store path per variant.  TMA bulk tensor stores from 128-byte-
+// Epilogue store path per mode.  TMA bulk tensor stores from 128-byte-
 // swizzled staging need 64 KB of shared memory, which leaves room for 3
 // pipeline slots at BN 256 instead of 4.  Measured on GB300 at the 17-task
-// ViT-B step: they pay for the weight gradients (always-full tiles, write-
-// bound) and for FC1 + GELU (two outputs per tile); FC2, dX and dA + GELU'
-// (which also writes two outputs, dH and its residual, but reads H) are
-// faster with 4 slots and masked st.global.
+// ViT-B step, they pay for the weight gradients (always-full tiles, write-
+// bound) only; every row-mode GEMM -- FC1 + GELU and dA + GELU' with their two
+// outputs included -- is faster with 4 slots and row-masked st.global (FC1:
+// 0.485 ms against 0.492 ms with TMA stores).
 template <int MODE, int EPI>
 struct UseTmaStore {
-    static constexpr bool value = MODE == 1 || EPI == 1;
+    static constexpr bool value = MODE == 1;
 };
 
 template <int BN, int MODE, int EPI>
@@ -667,154 +667,6 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
                 }
                 ++nstore;
             }
-        }
-        if (lane == 0) bulk_wait_all();
-        __syncwarp();
-    } else if (S::TMA_EPI) {
-        // ------------------------------------------------------------ epilogue (row mode, TMA stores)
-        // Warps 2..9.  Warps w and w+4 share TMEM lane quarter q = w & 3 (rows
-        // 32q..32q+31 of the tile) and split its BN columns in halves; each
-        // thread owns one row.  Columns are processed in 32-wide sub-chunks
-        // (tcgen05.ld, fused GELU / GELU') and staged as 64-wide chunks in a
-        // 128-byte-swizzled tile; a warp whose 32 rows are all valid stores a
-        // chunk with one TMA bulk tensor store, a partial warp stores its valid
-        // rows with 16-byte st.global.  Two staging buffers per warp; a buffer
-        // is rewritten only after the bulk store that last used it has read it.
-        const int ew = warp - 2;
-        const int q = warp & 3;
-        const int half = ew >> 2;
-        constexpr int COLS = BN / 2;
-        constexpr int NSC = COLS / 32;  // 32-column sub-chunks per warp
-        constexpr int NOUT = (EPI == EPI_GELU || EPI == EPI_DGELU) ? 2 : 1;
-        uint8_t *stg = epi_base + ew * EPI_WARP_BYTES_TMA;
-        const bool tanh_form = args.gelu_tanh != 0;
-        const int sub_r = lane >> 3, sub_c = lane & 7;  // read-back mapping: 4 rows x 8 x 16 B
-        uint4 hcur[4], hnxt[4];
-        auto load_h = [&](const Tile &tl, int sc, uint4 (&dst)[4]) {
-            const int r0 = tl.m_blk * BM + q * 32;
-            if (r0 + lane < tl.rows_valid) {
-                const uint4 *src = reinterpret_cast<const uint4 *>(
-                    args.aux + (long long)tl.gr * args.sAux + (long long)(r0 + lane) * args.ldd +
-                    tl.n_blk * BN + half * COLS + sc * 32);
-#pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
-            } else {
-#pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = make_uint4(0, 0, 0, 0);
-            }
-        };
-        auto write_sw = [&](uint8_t *buf, int cbase, const float *vv) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int j = cbase + i;
-                *reinterpret_cast<uint4 *>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                    f32_to_bf16x8(vv + i * 8);
-            }
-        };
-        auto flush = [&](uint8_t *buf, const CUtensorMap *map, __nv_bfloat16 *base, int col,
-                         int row0, int g, int nvalid) {
-            fence_proxy_async();
-            __syncwarp();
-            if (nvalid == 32) {
-                if (lane == 0) {
-                    tma_store_3d(map, smem_u32(buf), col, row0, g);
-                    bulk_commit();
-                }
-            } else {
-#pragma unroll
-                for (int i = 0; i < 8; ++i) {
-                    const int r = i * 4 + sub_r;
-                    if (r < nvalid)
-                        *reinterpret_cast<uint4 *>(base + (long long)r * args.ldd + sub_c * 8) =
-                            *reinterpret_cast<const uint4 *>(buf + r * 128 + ((sub_c ^ (r & 7)) << 4));
-                }
-                if (lane == 0) bulk_commit();  // empty group: keeps the buffer accounting uniform
-            }
-            __syncwarp();
-        };
-        int nstore = 0;
-        int it = 0;
-        Tile t = decode_tile<MODE>(args, prefix, blockIdx.x < total ? blockIdx.x : 0);
-        if (EPI == EPI_DGELU && blockIdx.x < total) load_h(t, 0, hcur);
-        for (int u = blockIdx.x; u < total; u += gridDim.x, ++it) {
-            const bool have_next = u + (int)gridDim.x < total;
-            const Tile tn = decode_tile<MODE>(args, prefix, have_next ? u + gridDim.x : u);
-            const int acc = it & 1;
-            const uint32_t aph = (uint32_t)((it >> 1) & 1);
-            if (!wait_phase(bar_tfull(acc), aph, abort_flag, args.status)) break;
-            tc_fence_after();
-            const int row0 = t.m_blk * BM + q * 32;  // this warp's first row in the group
-            int nvalid = t.rows_valid - row0;
-            nvalid = nvalid < 0 ? 0 : (nvalid > 32 ? 32 : nvalid);
-            const int colw = t.n_blk * BN + half * COLS;
-            const long long gofs = (long long)t.gr * args.sD + (long long)row0 * args.ldd + colw;
-            const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
-                                  (uint32_t)(acc * BN + half * COLS);
-            uint8_t *bufD = stg, *bufA = stg + 4096;
-            for (int sc = 0; sc < NSC; ++sc) {
-                if (EPI == EPI_DGELU) {
-                    if (sc + 1 < NSC) load_h(t, sc + 1, hnxt);
-                    else if (have_next) load_h(tn, 0, hnxt);
-                }
-                if (nvalid > 0) {
-                    if ((sc & 1) == 0) {  // a new 64-wide chunk: pick and free its buffer(s)
-                        if (NOUT == 2) {
-                            if (lane == 0 && nstore >= 1) bulk_wait_read0();
-                        } else {
-                            bufD = stg + (nstore & 1) * 4096;
-                            if (lane == 0 && nstore >= 2) bulk_wait_read1();
-                        }
-                        __syncwarp();
-                    }
-                    float v[32];
-                    if (t.kblocks > 0) {
-                        uint32_t r[32];
-                        tmem_ld32(trow + sc * 32, r);
-                        tmem_ld_wait();
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
-                    } else {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = 0.0f;
-                    }
-                    if (EPI == EPI_DGELU) {
-#pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float hv[8];
-                            bf16x8_to_f32(hcur[i], hv);
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_fast(hv[e], tanh_form);
-                        }
-                    }
-                    write_sw(bufD, (sc & 1) * 4, v);
-                    if (EPI == EPI_GELU) {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = gelu_fast(v[i], tanh_form);
-                        write_sw(bufA, (sc & 1) * 4, v);
-                    } else if (EPI == EPI_DGELU) {
-#pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] -= __bfloat162float(__float2bfloat16_rn(v[i]));
-                        write_sw(bufA, (sc & 1) * 4, v);
-                    }
-                    if ((sc & 1) == 1) {
-                        const int c64 = (sc >> 1) * 64;
-                        flush(bufD, &tmD, args.D + gofs + c64, colw + c64, row0, t.gr, nvalid);
-                        ++nstore;
-                        if (NOUT == 2) {
-                            flush(bufA, &tmD2, args.D2 + gofs + c64, colw + c64, row0, t.gr, nvalid);
-                            ++nstore;
-                        }
-                    }
-                }
-                if (EPI == EPI_DGELU) {
-#pragma unroll
-                    for (int i = 0; i < 4; ++i) hcur[i] = hnxt[i];
-                }
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar_tempty(acc));
-            t = tn;
         }
         if (lane == 0) bulk_wait_all();
         __syncwarp();
@@ -1431,11 +1283,7 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
         a.compact = sl.compact;
     }
     long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
-    CUtensorMap md = {}, md2 = {};  // output maps: 64 x 32 store boxes over [G, C, N]
-    if (UseTmaStore<MODE_ROW, EPI>::value) {
-        if (!make_map(&md, D, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
-        if (D2 && !make_map(&md2, D2, N, C, G, 32, (uint64_t)a.sD)) return VMOE_ERR_CUDA;
-    }
+    const CUtensorMap md = {}, md2 = {};  // row mode stores with st.global: no output maps
     return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name)
                 : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name);
 }
