@@ -48,6 +48,13 @@ CASES = {
                            dtype="bf16", capacity=1),
     "one_token": Config("one_token", 68, T=3, N=1, d=256, f=128, E=4, k=2, cf=1.0,
                         dtype="bf16"),
+    # E = 32 takes the tcgen05 dW_r kernel: N = 131 gives the two ranks of a
+    # cluster 65 and 66 tokens (a full and a partial k-block each), d = 256 two slices
+    "bf16_e32_ragged": Config("bf16_e32_ragged", 69, T=3, N=131, d=256, f=128, E=32, k=2, cf=1.25,
+                              dtype="bf16", bias="drift"),
+    # one token: the first rank of every cluster has no tokens at all
+    "bf16_e32_one_token": Config("bf16_e32_one_token", 70, T=2, N=1, d=128, f=128, E=32, k=2,
+                                 cf=1.0, dtype="bf16"),
 }
 
 
