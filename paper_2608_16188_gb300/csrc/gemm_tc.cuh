@@ -1330,7 +1330,13 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
         a.crow = sl.crow;
         a.compact = sl.compact;
     }
-    if (ksplit && N % BSTAT_BN == 0 && C <= 2 * BK) {  // every group fits one resident B tile
+    // Resident B when every group fits one B tile (C <= 128) but is not tiny: with
+    // C <= 32 a unit has almost no MMA work to hide its B reload behind, and the
+    // streaming kernel, which pipelines across tiles, is faster (measured at the
+    // Zipf-skewed workload, C = 25: 0.770 against 0.904 ms; at C = 124 the
+    // resident-B kernel wins, 0.566 against 0.749 ms).
+    constexpr int BSTAT_MIN_C = 32;
+    if (ksplit && N % BSTAT_BN == 0 && C <= 2 * BK && C > BSTAT_MIN_C) {
         using SB = BStatShape<BSTAT_BN, true, BSTAT_BUFS>;
         CUtensorMap mbs;
         if (!make_map_chunked(&mbs, act2, N, b_rows, b_outer, 64, BSTAT_BN / 64)) return VMOE_ERR_CUDA;
