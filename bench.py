@@ -92,15 +92,19 @@ def model_counts(cfg, loads):
     }
 
 
-def traffic_record(kernel):
+def traffic_record(kernel, workload, path=None):
     """DRAM bytes per launch of `kernel` from the committed ncu summary
-    (profiles/dram_traffic.json), if the kernel's source files still hash to the
-    value recorded with the counters; else None."""
+    (profiles/dram_traffic.json), if it was captured on `workload` and the
+    kernel's source files still hash to the value recorded with the counters;
+    else None."""
     import hashlib
-    path = os.path.join(ROOT, "profiles", "dram_traffic.json")
+    path = path or os.path.join(ROOT, "profiles", "dram_traffic.json")
     try:
         with open(path) as fh:
-            rec = json.load(fh)["kernels"][kernel]
+            data = json.load(fh)
+        if data.get("workload") != workload:
+            return None
+        rec = data["kernels"][kernel]
         h = hashlib.sha256()
         for f in rec["source_files"]:
             with open(os.path.join(ROOT, f), "rb") as fh:
@@ -351,13 +355,19 @@ def run_ours(args, cfg, rank, world, local_rank):
     counts = model_counts(cfg, loads)
     peaks = load_peaks()
     kstats = {}
+    # the committed DRAM records hold for their workload at its full task count only
+    # (a --tasks prefix keeps the name but not the sizes)
+    traffic_key = cfg.name if cfg.T == workloads.CONFIGS[cfg.name].T else None
     for name, ms_list in per_kernel.items():
         avg = sum(ms_list) / len(ms_list)
         by, fl = counts.get(name, (0, 0.0))
         launches_per_step = len(ms_list) / trace_steps
+        tr = traffic_record(name, traffic_key)
         kstats[name] = {"launches": len(ms_list), "ms_avg": round(avg, 5),
                         "share": 0.0,
                         "gb_s": round(by / (avg * 1e-3) / 1e9, 1) if by else None,
+                        # on the measured DRAM traffic (the committed ncu launch list)
+                        "dram_gb_s": round(tr / (avg * 1e-3) / 1e9, 1) if tr else None,
                         "tflop_s": round(fl / (avg * 1e-3) / 1e12, 2) if fl else None,
                         "launches_per_step": launches_per_step}
     busy = sum(v["ms_avg"] * v["launches"] for v in kstats.values())
@@ -370,7 +380,7 @@ def run_ours(args, cfg, rank, world, local_rank):
     roofline = {"kernel": dom, "bound": "hbm", "achieved": round(achieved, 1),
                 "peak": peaks["hbm_gbs"], "unit": "GB/s",
                 "frac": round(achieved / peaks["hbm_gbs"], 4),
-                "traffic": traffic_record(dom),
+                "traffic": traffic_record(dom, traffic_key),
                 "algorithmic_bytes_per_launch": dom_bytes,
                 "peak_source": peaks["source"] + " (MEASURED_PEAKS.json hbm_gbs)"}
     rb_stats = {}
@@ -394,7 +404,7 @@ def run_ours(args, cfg, rank, world, local_rank):
             "roofline": {"kernel": rb_dom, "bound": "hbm", "achieved": rb_ach,
                          "peak": peaks["hbm_gbs"], "unit": "GB/s",
                          "frac": round(rb_ach / peaks["hbm_gbs"], 4),
-                         "traffic": traffic_record(rb_dom),
+                         "traffic": traffic_record(rb_dom, traffic_key),
                          "peak_source": peaks["source"] + " (MEASURED_PEAKS.json hbm_gbs)"},
             "step_with_router_bwd_tokens_per_s": round(
                 job_tokens_per_s(cfg.T * cfg.N, world, ms_step + rb_ms), 1),
