@@ -16,15 +16,17 @@ namespace vmoe {
 static __device__ int g_status_word = 0;
 
 int *device_status_word() {
-    static int *addr[64] = {nullptr};
+    static std::atomic<int *> addr[64];  // per device; the same value from every thread
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
-    if (!addr[dev]) {
+    int *a = addr[dev].load(std::memory_order_acquire);
+    if (!a) {
         void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return nullptr;
-        addr[dev] = static_cast<int *>(p);
+        a = static_cast<int *>(p);
+        addr[dev].store(a, std::memory_order_release);
     }
-    return addr[dev];
+    return a;
 }
 
 bool pdl_enabled() {
@@ -36,15 +38,17 @@ bool pdl_enabled() {
 }
 
 int num_sms() {
-    static int sms[64] = {0};
+    static std::atomic<int> sms[64];  // per device; the same value from every thread
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 1;
-    if (!sms[dev]) {
+    int n = sms[dev].load(std::memory_order_relaxed);
+    if (!n) {
         int v = 0;
         cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev);
-        sms[dev] = v > 0 ? v : 1;
+        n = v > 0 ? v : 1;
+        sms[dev].store(n, std::memory_order_relaxed);
     }
-    return sms[dev];
+    return n;
 }
 
 // ---------------------------------------------------------------------------

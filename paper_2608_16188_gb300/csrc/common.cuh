@@ -5,6 +5,9 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+#include <mutex>
+
 #include <utility>
 
 #include "vmoe.h"
@@ -97,6 +100,23 @@ int launch_router_bwd(const Dims &p, const void *x, const float *w_router, const
 
 // ---------------------------------------------------------------------------
 // Device helpers.
+
+// Raises `kern`'s dynamic shared-memory limit on the current device to at
+// least `bytes`, never lowering it, so that concurrent host threads launching
+// it with different sizes all stay within the limit.  `limit` caches the value
+// set per device (up to 64 devices).
+inline int raise_smem_limit(const void *kern, std::atomic<int> (&limit)[64], int bytes) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
+    if (limit[dev].load(std::memory_order_acquire) >= bytes) return VMOE_OK;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    if (limit[dev].load(std::memory_order_relaxed) >= bytes) return VMOE_OK;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes) != cudaSuccess)
+        return VMOE_ERR_CUDA;
+    limit[dev].store(bytes, std::memory_order_release);
+    return VMOE_OK;
+}
 
 // Programmatic dependent launch (see launch_kernel); both are no-ops in a
 // kernel launched without the attribute.

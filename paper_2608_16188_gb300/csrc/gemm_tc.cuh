@@ -1179,15 +1179,8 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
            cudaStream_t s, const char *name) {
     using S = Shape<BN, MODE, EPI>;
     auto kern = grouped_gemm_kernel<BN, MODE, A_MN, B_MN, EPI>;
-    static uint64_t attr_done = 0;  // one bit per device
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !(attr_done >> dev & 1ull)) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)S::SMEM_BYTES) != cudaSuccess)
-            return VMOE_ERR_CUDA;
-        attr_done |= 1ull << dev;
-    }
+    static std::atomic<int> smem_limit[64];
+    if (const int st = raise_smem_limit((const void *)kern, smem_limit, (int)S::SMEM_BYTES)) return st;
     if (max_tiles <= 0) return VMOE_OK;
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
@@ -1202,15 +1195,8 @@ int launch_bstat(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap
                  const Args &a, long long units, cudaStream_t s, const char *name) {
     using S = BStatShape<BN, KSPLIT, B_BUFS>;
     auto kern = wgrad_bstat_kernel<BN, KSPLIT, B_BUFS>;
-    static uint64_t attr_done = 0;  // one bit per device
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev < 64 && !(attr_done >> dev & 1ull)) {
-        if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)S::SMEM_BYTES) != cudaSuccess)
-            return VMOE_ERR_CUDA;
-        attr_done |= 1ull << dev;
-    }
+    static std::atomic<int> smem_limit[64];
+    if (const int st = raise_smem_limit((const void *)kern, smem_limit, (int)S::SMEM_BYTES)) return st;
     if (units <= 0) return VMOE_OK;
     long long grid = units < num_sms() ? units : num_sms();
     trace_before(s, name);

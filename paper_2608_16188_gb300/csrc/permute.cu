@@ -207,10 +207,10 @@ int launch_dispatch(const Dims &p, const void *src, const float *weight, const i
 // Persistent grid: at most as many CTAs as fit on the GPU at once.
 template <typename T, int KMAX>
 static unsigned combine_grid(long long blocks) {
-    static int per_sm[64];
+    static std::atomic<int> per_sm[64];  // per device; the same value from every thread
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return (unsigned)blocks;
-    if (per_sm[dev] < 1) {
+    if (per_sm[dev].load(std::memory_order_relaxed) < 1) {
         int v = 0;
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, combine_kernel<T, KMAX>, PM_THREADS, 0) !=
                 cudaSuccess || v < 1)

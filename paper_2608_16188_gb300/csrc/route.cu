@@ -303,15 +303,8 @@ int launch_mma_router(const Dims &p, const __nv_bfloat16 *x, const float *wr, co
     constexpr int NP = NB * 8;
     size_t smem = (size_t)RM_TOK * RM_XP * 2 + (size_t)3 * NP * RM_XP * 2 + (size_t)RM_TOK * (p.E + 1) * 4;
     if (smem > 227 * 1024) return VMOE_ERR_UNSUPPORTED;
-    static int attr_bytes[64];  // per device: the largest size set so far
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
-    if (attr_bytes[dev] < (int)smem) {
-        if (cudaFuncSetAttribute(route_mma_kernel<NB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem) != cudaSuccess)
-            return VMOE_ERR_CUDA;
-        attr_bytes[dev] = (int)smem;
-    }
+    static std::atomic<int> smem_limit[64];  // the size depends on E
+    if (const int st = raise_smem_limit((const void *)route_mma_kernel<NB>, smem_limit, (int)smem)) return st;
     dim3 grid((p.N + RM_TOK - 1) / RM_TOK, p.T);
     trace_before(s, "route_topk");
     const int st = launch_kernel(route_mma_kernel<NB>, grid, dim3(RM_THREADS), smem, s, p, x, wr, bias,
@@ -404,12 +397,9 @@ int launch_topk(const Dims &p, const TX *x, const float *wr, const float *bias, 
                 int32_t *idx, float *gate, cudaStream_t s) {
     constexpr int TOK = 16 * RT_THREADS / ECH;
     size_t smem = sizeof(float) * ((size_t)RT_KC * TOK + (size_t)RT_KC * ECH + (size_t)TOK * (p.E + 1));
-    static bool attr_set = false;  // per instantiation; same value on every device
-    if (!attr_set) {
-        cudaFuncSetAttribute(route_topk_kernel<TX, ECH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             96 * 1024);
-        attr_set = true;
-    }
+    static std::atomic<int> smem_limit[64];
+    if (const int st = raise_smem_limit((const void *)route_topk_kernel<TX, ECH>, smem_limit, (int)smem))
+        return st;
     dim3 grid((p.N + TOK - 1) / TOK, p.T);
     trace_before(s, "route_topk");
     route_topk_kernel<TX, ECH><<<grid, RT_THREADS, smem, s>>>(p, x, wr, bias, logits, idx, gate,
@@ -424,14 +414,10 @@ int launch_scan(const Dims &p, const int32_t *idx, int32_t *slot, int32_t *load,
     const size_t smem_small = sizeof(int) * (size_t)(CS_THREADS / 32) * p.E;
     const size_t smem_big = smem_small + sizeof(int) * 2 * total;
     if (smem_big <= 96 * 1024) {
-        static uint64_t attr_done = 0;
-        int dev = 0;
-        cudaGetDevice(&dev);
-        if (dev < 64 && !(attr_done >> dev & 1ull)) {
-            cudaFuncSetAttribute(capacity_scan_kernel<true, CS_THREADS>,
-                                 cudaFuncAttributeMaxDynamicSharedMemorySize, 96 * 1024);
-            attr_done |= 1ull << dev;
-        }
+        static std::atomic<int> smem_limit[64];
+        if (const int st = raise_smem_limit((const void *)capacity_scan_kernel<true, CS_THREADS>, smem_limit,
+                                            (int)smem_big))
+            return st;
         return launch_kernel(capacity_scan_kernel<true, CS_THREADS>, dim3(p.T), dim3(CS_THREADS), smem_big,
                              s, p, idx, slot, load);
     }

@@ -783,23 +783,21 @@ int launch_grad(const Dims &p, const float *wr, const float *logits, const int32
                 const float *gate, const int32_t *slot, const T *dy, const T *ye, float *dgate,
                 float *dlogits, T *dx, size_t smem, cudaStream_t s) {
     auto kern = router_grad_kernel<T, KMAX, WSMEM>;
-    // attribute and occupancy per (device, shared-memory size), set up once
-    static int cached_smem[64];
-    static int cached_per_sm[64];
+    // attribute and occupancy per (device, shared-memory size)
+    static std::atomic<int> smem_limit[64];
+    static std::atomic<uint64_t> occupancy[64];  // per device: (smem << 32) | CTAs per SM
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
-    int per_sm = cached_per_sm[dev];
-    if (per_sm < 1 || cached_smem[dev] != (int)smem) {
-        if (smem > 48 * 1024 &&
-            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-                cudaSuccess)
-            return VMOE_ERR_CUDA;
+    if (smem > 48 * 1024)
+        if (const int st = raise_smem_limit((const void *)kern, smem_limit, (int)smem)) return st;
+    const uint64_t o = occupancy[dev].load(std::memory_order_relaxed);
+    int per_sm = (int)(o & 0xffffffffu);
+    if (per_sm < 1 || (o >> 32) != (uint64_t)smem) {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, RG_THREADS, smem) !=
                 cudaSuccess ||
             per_sm < 1)
             return VMOE_ERR_CUDA;
-        cached_smem[dev] = (int)smem;
-        cached_per_sm[dev] = per_sm;
+        occupancy[dev].store(((uint64_t)smem << 32) | (uint32_t)per_sm, std::memory_order_relaxed);
     }
     const long long tokens = (long long)p.T * p.N;
     long long grid = (long long)per_sm * num_sms();
@@ -815,22 +813,20 @@ int launch_grad_fast(const Dims &p, const float *wr, const float *logits, const 
                      const __nv_bfloat16 *ye, float *dgate, float *dlogits, __nv_bfloat16 *dx,
                      size_t smem, cudaStream_t s) {
     auto kern = router_grad_fast_kernel<NCH, KMAX, WSMEM>;
-    static int cached_smem[64];
-    static int cached_per_sm[64];
+    static std::atomic<int> smem_limit[64];
+    static std::atomic<uint64_t> occupancy[64];  // per device: (smem << 32) | CTAs per SM
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
-    int per_sm = cached_per_sm[dev];
-    if (per_sm < 1 || cached_smem[dev] != (int)smem) {
-        if (smem > 48 * 1024 &&
-            cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-                cudaSuccess)
-            return VMOE_ERR_CUDA;
+    if (smem > 48 * 1024)
+        if (const int st = raise_smem_limit((const void *)kern, smem_limit, (int)smem)) return st;
+    const uint64_t o = occupancy[dev].load(std::memory_order_relaxed);
+    int per_sm = (int)(o & 0xffffffffu);
+    if (per_sm < 1 || (o >> 32) != (uint64_t)smem) {
         if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, RG_THREADS, smem) !=
                 cudaSuccess ||
             per_sm < 1)
             return VMOE_ERR_CUDA;
-        cached_smem[dev] = (int)smem;
-        cached_per_sm[dev] = per_sm;
+        occupancy[dev].store(((uint64_t)smem << 32) | (uint32_t)per_sm, std::memory_order_relaxed);
     }
     const long long tokens = (long long)p.T * p.N;
     long long grid = (long long)per_sm * num_sms();

@@ -293,15 +293,9 @@ router_dw_tc_kernel(const __grid_constant__ CUtensorMap tmX, Dims p, const float
 template <int E>
 int launch_rw(const Dims &p, const __nv_bfloat16 *x, const float *dl, float *dw, float *dbias, cudaStream_t s) {
     using S = RwShape<E>;
-    static uint64_t attr_done = 0;  // one bit per device
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return VMOE_ERR_CUDA;
-    if (!(attr_done >> dev & 1ull)) {
-        if (cudaFuncSetAttribute(router_dw_tc_kernel<E>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)S::SMEM) != cudaSuccess)
-            return VMOE_ERR_CUDA;
-        attr_done |= 1ull << dev;
-    }
+    static std::atomic<int> smem_limit[64];
+    if (const int st = raise_smem_limit((const void *)router_dw_tc_kernel<E>, smem_limit, (int)S::SMEM))
+        return st;
     CUtensorMap mx;  // x [T][N][d] as {64, N, d / 64, T}: 64-token boxes of two 64-wide d chunks
     if (!make_map_chunked(&mx, x, p.d, p.N, p.T, RW_KB, 2)) return VMOE_ERR_CUDA;
     dim3 grid(RW_RS, p.d / 128, p.T);
