@@ -33,10 +33,15 @@
  *  - Errors: arguments are checked on the host before any launch; an invalid
  *    argument returns VMOE_ERR_INVALID and an unsupported shape
  *    VMOE_ERR_UNSUPPORTED, in both cases with nothing launched.  A failed
- *    launch returns VMOE_ERR_CUDA.  Device data (indices, loads) is trusted:
- *    indices out of range are undefined behaviour.
+ *    launch returns VMOE_ERR_CUDA.  Device data is trusted: loads are clamped
+ *    to [0, C], and expert indices or slots out of range are undefined
+ *    behaviour.
  *  - Determinism: results are bitwise reproducible run to run (no atomics in
  *    any reduction, fixed summation orders).
+ *  - Host threads: entry points may be called from several host threads at
+ *    once, each with its own stream and arrays; the kernel trace is kept per
+ *    host thread.  The exception is vmoe_expert_bwd_static_scratch, whose
+ *    calls share one device array (see there).
  *  - Dtypes: x, dY, weights and all activations use p->dtype (fp32 or bf16);
  *    W_r, bias, logits and gates are always fp32.  bf16 contractions
  *    accumulate in fp32 on the tcgen05 tensor cores; fp32 runs on CUDA cores.
