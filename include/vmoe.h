@@ -195,14 +195,21 @@ int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const 
  *   Arguments, layouts and results are those of vmoe_expert_bwd.  The dH
  *   scratch is a 64 MiB array compiled into the library, which every GPU that
  *   loads the library holds until the process exits; the call itself allocates
- *   nothing.  A problem whose vmoe_expert_bwd_workspace_size exceeds
- *   VMOE_STATIC_SCRATCH_BYTES returns VMOE_ERR_UNSUPPORTED with nothing
- *   launched.  The first call on a device looks up the array's device address
- *   (cudaGetSymbolAddress) with that device current; make that first call
- *   before any stream capture.  Every call on a device shares the one array,
- *   which keeps whatever the last call left in it, so calls whose kernels
- *   overlap on the GPU (other streams, other host threads) race and corrupt
- *   each other's dH; issue them in order on one stream. */
+ *   nothing.  When vmoe_expert_bwd_workspace_size(p) <= VMOE_STATIC_SCRATCH_BYTES,
+ *   dH of every group fits and the call is asynchronous like vmoe_expert_bwd.
+ *   Otherwise a bf16 problem runs in slices planned to fit the array (as
+ *   vmoe_expert_bwd with a smaller workspace): that path reads `load` back to
+ *   the host and synchronises `cuda_stream`.  The call returns
+ *   VMOE_ERR_UNSUPPORTED, with nothing launched, only when even
+ *   vmoe_expert_bwd_min_workspace_size(p) exceeds the array: an fp32 problem
+ *   whose dH is larger than the array, or a bf16 problem one of whose groups
+ *   alone does not fit.  The first call on a device looks up the array's
+ *   device address (cudaGetSymbolAddress) with that device current and caches
+ *   it; make that first call before any stream capture.  Every call on a
+ *   device shares the one array, which keeps whatever the last call left in
+ *   it, so calls whose kernels overlap on the GPU (other streams, other host
+ *   threads) race and corrupt each other's dH; issue them in order on one
+ *   stream. */
 int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void *xe, const void *h,
                                    const void *a, const void *w1, const void *w2, const void *dye,
                                    const int32_t *load, void *dxe, void *dw1, void *dw2,

@@ -37,6 +37,22 @@ bool pdl_enabled() {
     return on;
 }
 
+bool pair_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("VMOE_PAIR");
+        return !(v && v[0] == '0');
+    }();
+    return on;
+}
+
+bool row_pair_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("VMOE_ROW_PAIR");
+        return v && v[0] == '1';
+    }();
+    return on;
+}
+
 int num_sms() {
     static std::atomic<int> sms[64];  // per device; the same value from every thread
     int dev = 0;

@@ -9,7 +9,10 @@
 // scratch in a fixed array that lives in the library itself.
 //
 // When dH for every group does not fit, the bf16 backward runs in slices of
-// groups planned to fit the array (vmoe_expert_bwd with a smaller workspace).
+// groups planned to fit the array (vmoe_expert_bwd with a smaller workspace),
+// which reads the loads back to the host and synchronises the stream.  Only a
+// problem whose smallest workspace (one group's dH, or all of an fp32
+// problem's dH) exceeds the array is refused.
 //
 // The array is a file-scope __device__ variable: every GPU that loads the
 // library holds VMOE_STATIC_SCRATCH_BYTES of it until the process exits.  In
@@ -23,7 +26,9 @@ namespace {
 static __device__ __align__(256) unsigned char g_bwd_scratch[VMOE_STATIC_SCRATCH_BYTES];
 
 constexpr int kMaxDevices = 64;
-void *g_scratch_addr[kMaxDevices] = {nullptr};
+// Per-device cache of the array's device address.  Host threads may call
+// concurrently; each stores the same value, published with release order.
+std::atomic<void *> g_scratch_addr[kMaxDevices];
 
 }  // namespace
 
@@ -39,13 +44,13 @@ extern "C" int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void 
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return VMOE_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices) return VMOE_ERR_UNSUPPORTED;
-    if (g_scratch_addr[dev] == nullptr) {  // first call on this device: resolve the address
-        void *addr = nullptr;
+    void *addr = g_scratch_addr[dev].load(std::memory_order_acquire);
+    if (addr == nullptr) {  // first call on this device: resolve the address
         if (cudaGetSymbolAddress(&addr, g_bwd_scratch) != cudaSuccess || addr == nullptr)
             return VMOE_ERR_CUDA;
-        g_scratch_addr[dev] = addr;
+        g_scratch_addr[dev].store(addr, std::memory_order_release);
     }
     // dH needs no clearing: the backward writes every row it later reads.
-    return vmoe_expert_bwd(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2, g_scratch_addr[dev],
+    return vmoe_expert_bwd(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2, addr,
                            VMOE_STATIC_SCRATCH_BYTES, cuda_stream);
 }

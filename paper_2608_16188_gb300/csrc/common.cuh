@@ -44,6 +44,12 @@ inline int launch_result() {
 // On by default; the environment variable VMOE_PDL=0 turns it off.
 bool pdl_enabled();  // abi.cu
 
+// The SM-pair (cta_group::2) grouped GEMMs (abi.cu): the weight-gradient
+// kernel, on unless VMOE_PAIR=0 in the environment; the row-mode kernel for
+// groups above 128 rows, off unless VMOE_ROW_PAIR=1.
+bool pair_enabled();
+bool row_pair_enabled();
+
 template <typename... KArgs, typename... Args>
 int launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
                   Args &&...args) {

@@ -1170,8 +1170,10 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, 
 // box_chunks, 1} box then lands in shared memory chunk-major -- box_chunks
 // tiles of box_rows x 128 bytes (128-byte swizzle) -- which is the MN-major
 // operand layout, in one copy instead of one per chunk.
+// outer_stride_elems: elements from one outer index to the next (0: rows x mn).
 bool make_map_chunked(CUtensorMap *map, const void *base, uint64_t mn, uint64_t rows,
-                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks);
+                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks,
+                      uint64_t outer_stride_elems = 0);
 
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
 int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
@@ -1226,116 +1228,6 @@ inline Args base_args(const Dims &p, const int32_t *load) {
     a.gelu_tanh = (p.flags & VMOE_GELU_TANH) != 0;
     a.status = device_status_word();
     return a;
-}
-
-// Row-mode GEMM: D[g][C rows][N] = act[g][C][K] * B, B MN-major ([K][N]) or
-// K-major ([N][K]).
-// sD / sAux / sAct: group strides (elements) of D and D2, of aux, and of act;
-// 0 means the dense [G, C, width] layout.
-template <int EPI, bool B_MN>
-int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16 *w, int N,
-             const int32_t *load, __nv_bfloat16 *D, __nv_bfloat16 *D2, const __nv_bfloat16 *aux,
-             cudaStream_t s, const char *name, long long sD = 0, long long sAux = 0,
-             long long sAct = 0, const Slice &sl = Slice()) {
-    const int G = p.G(), C = p.C;
-    const bool wide = N % 256 == 0;
-    const int BN = wide ? 256 : 128;
-    CUtensorMap ma, mb;
-    TailMaps mat;
-    const bool cmpa = (sl.compact & CMP_A) != 0;
-    auto amap = [&](CUtensorMap *m, uint32_t box) {
-        return cmpa ? make_map(m, act, K, (uint64_t)sl.rows, 1, box)
-                    : make_map(m, act, K, C, G, box, (uint64_t)sAct);
-    };
-    if (!amap(&ma, 128) || !amap(&mat.a[0], 64) || !amap(&mat.a[1], 32) || !amap(&mat.a[2], 16))
-        return VMOE_ERR_CUDA;
-    bool okb = B_MN ? make_map_chunked(&mb, w, N, K, G, 64, BN / 64) : make_map(&mb, w, K, N, G, BN);
-    if (!okb) return VMOE_ERR_CUDA;
-    Args a = base_args(p, load);
-    a.N = N;
-    a.K_fixed = K;
-    a.tiles_n = N / BN;
-    a.tiles_m = (C + BM - 1) / BM;
-    a.D = D;
-    a.D2 = D2;
-    a.aux = aux;
-    a.sD = sD ? sD : (long long)C * N;
-    a.sAux = sAux ? sAux : (long long)C * N;
-    a.ldd = N;
-    if (sl.n > 0) {
-        a.G = sl.n;
-        a.glist = sl.glist;
-        a.crow = sl.crow;
-        a.compact = sl.compact;
-    }
-    long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
-    const CUtensorMap md = {}, md2 = {};  // row mode stores with st.global: no output maps
-    return wide ? launch<256, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name)
-                : launch<128, MODE_ROW, false, B_MN, EPI>(ma, mb, md, md2, mat, a, max_tiles, s, name);
-}
-
-// Weight-gradient GEMM: D[g][M][N] = act1[g][C][M]^T * act2[g][C][N], summed
-// over each group's load[g] rows; both operands MN-major.
-// ksplit: act2 is [G, 2C, N] -- a bf16 part in rows [0, C) and its residual in
-// rows [C, 2C) -- and D = act1^T (hi + lo), the K loop running over both halves.
-inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __nv_bfloat16 *act2,
-                      int N, const int32_t *load, __nv_bfloat16 *D, cudaStream_t s,
-                      const char *name, bool ksplit = false, const Slice &sl = Slice()) {
-    const int G = p.G(), C = p.C;
-    const bool wide = N % 256 == 0;
-    const int BN = wide ? 256 : 128;
-    const bool cmpb = (sl.compact & CMP_B) != 0;
-    // B: per-group slabs of C (with ksplit 2C) rows, or the compact buffer
-    const uint64_t b_rows = cmpb ? (uint64_t)sl.rows : (uint64_t)(ksplit ? 2 * C : C);
-    const uint64_t b_outer = cmpb ? 1 : (uint64_t)G;
-    CUtensorMap ma, mb, md;
-    TailMaps mt;  // the last k-block's boxes of 16, 32 and 48 K rows
-    // b_chunks: the B tile's 64-column chunks (the kernel's BN / 64)
-    auto tail_maps = [&](int b_chunks) {
-        for (int i = 0; i < 3; ++i)
-            if (!make_map_chunked(&mt.a[i], act1, M, C, G, 16 * (i + 1), BM / 64) ||
-                !make_map_chunked(&mt.b[i], act2, N, b_rows, b_outer, 16 * (i + 1), b_chunks))
-                return false;
-        return true;
-    };
-    if (!make_map_chunked(&ma, act1, M, C, G, 64, BM / 64)) return VMOE_ERR_CUDA;
-    if (!make_map_chunked(&mb, act2, N, b_rows, b_outer, 64, BN / 64)) return VMOE_ERR_CUDA;
-    if (!make_map(&md, D, N, M, G, 32)) return VMOE_ERR_CUDA;  // 64 x 32 store boxes
-    Args a = base_args(p, load);
-    a.N = N;
-    a.M_fixed = M;
-    a.tiles_n = N / BN;
-    a.tiles_m = M / BM;
-    a.D = D;
-    a.sD = (long long)M * N;
-    a.ldd = N;
-    a.ksplit = ksplit ? 1 : 0;
-    if (sl.n > 0) {
-        a.G = sl.n;
-        a.glist = sl.glist;
-        a.crow = sl.crow;
-        a.compact = sl.compact;
-    }
-    // Resident B when every group fits one B tile (C <= 128) but is not tiny: with
-    // C <= 32 a unit has almost no MMA work to hide its B reload behind, and the
-    // streaming kernel, which pipelines across tiles, is faster (measured at the
-    // Zipf-skewed workload, C = 25: 0.770 against 0.904 ms; at C = 124 the
-    // resident-B kernel wins, 0.566 against 0.749 ms).
-    constexpr int BSTAT_MIN_C = 32;
-    if (ksplit && N % BSTAT_BN == 0 && C <= 2 * BK && C > BSTAT_MIN_C) {
-        using SB = BStatShape<BSTAT_BN, true, BSTAT_BUFS>;
-        CUtensorMap mbs;
-        if (!make_map_chunked(&mbs, act2, N, b_rows, b_outer, 64, BSTAT_BN / 64)) return VMOE_ERR_CUDA;
-        if (!tail_maps(BSTAT_BN / 64)) return VMOE_ERR_CUDA;
-        a.tiles_n = N / BSTAT_BN;
-        const int nch = (a.tiles_m + SB::MCH - 1) / SB::MCH;
-        const long long units = (long long)a.G * a.tiles_n * nch;
-        return launch_bstat<BSTAT_BN, true, BSTAT_BUFS>(ma, mbs, md, mt, a, units, s, name);
-    }
-    long long max_tiles = (long long)a.G * a.tiles_m * a.tiles_n;
-    const TailMaps unused{};  // the streaming kernel loads full k-blocks
-    return wide ? launch<256, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, unused, a, max_tiles, s, name)
-                : launch<128, MODE_WGRAD, true, true, EPI_STORE>(ma, mb, md, md, unused, a, max_tiles, s, name);
 }
 
 }  // namespace tc

@@ -5,12 +5,52 @@
 //   dW2:        dW2 = A^T dYe               (both MN-major, K = load)
 #include <vector>
 
-#include "gemm_tc.cuh"
+#include "gemm_tc2.cuh"
 
 namespace vmoe {
 
 int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
                 double budget, int32_t *order, int32_t *slice_start);  // planner.cu
+
+namespace tc {
+int pair_clusters(const void *kern, size_t smem) {
+    // per device and kernel: the kernels are few, a small table does
+    struct Entry {
+        std::atomic<const void *> kern;
+        std::atomic<int> n;
+    };
+    static Entry cache[64][8];
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+    for (auto &e : cache[dev])
+        if (e.kern.load(std::memory_order_acquire) == kern) return e.n.load(std::memory_order_relaxed);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(2 * (unsigned)num_sms());
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, kern, &cfg) != cudaSuccess || n <= 0) return 0;
+    static std::mutex mu;
+    std::lock_guard<std::mutex> lock(mu);
+    for (auto &e : cache[dev]) {
+        const void *k = e.kern.load(std::memory_order_relaxed);
+        if (k == kern) break;
+        if (k == nullptr) {
+            e.n.store(n, std::memory_order_relaxed);
+            e.kern.store(kern, std::memory_order_release);
+            break;
+        }
+    }
+    return n;
+}
+}  // namespace tc
 
 using namespace tc;
 

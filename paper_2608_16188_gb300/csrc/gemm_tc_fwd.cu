@@ -2,7 +2,7 @@
 // tcgen05 grouped GEMM:
 //   FC1 + GELU: H = Xe W1, A = GELU(H)   (A: Xe K-major; B: W1 [d,f] MN-major)
 //   FC2:        Ye = A W2                (A: A  K-major; B: W2 [f,d] MN-major)
-#include "gemm_tc.cuh"
+#include "gemm_tc2.cuh"
 
 namespace vmoe {
 namespace tc {
@@ -40,11 +40,13 @@ bool make_map(CUtensorMap *map, const void *base, uint64_t inner, uint64_t mid, 
 }
 
 bool make_map_chunked(CUtensorMap *map, const void *base, uint64_t mn, uint64_t rows,
-                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks) {
+                      uint64_t outer, uint32_t box_rows, uint32_t box_chunks,
+                      uint64_t outer_stride_elems) {
     EncodeTiledFn fn = encoder();
     if (!fn || mn % 64 != 0) return false;
     cuuint64_t dims[4] = {64, rows, mn / 64, outer};
-    cuuint64_t strides[3] = {mn * 2, 128, rows * mn * 2};  // bytes: row, chunk, group
+    // bytes: row, chunk, group
+    cuuint64_t strides[3] = {mn * 2, 128, (outer_stride_elems ? outer_stride_elems : rows * mn) * 2};
     cuuint32_t box[4] = {64, box_rows, box_chunks, 1};
     cuuint32_t estr[4] = {1, 1, 1, 1};
     CUresult r = fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(base), dims, strides,

@@ -2,9 +2,10 @@
 
 The grouped GEMMs load only a group's valid rows: row-mode A tiles load
 16 ceil(load / 16) rows as 64-, 32- and 16-row boxes, and the resident-B
-weight-gradient kernel loads a group's last k-block with a 16-, 32- or 48-row
-box.  Here every group of one launch has its own load, covering each residue
-(0, 1, 15-17, 31-33, ..., 127, 128 rows of a 128-row capacity), and every
+weight-gradient kernels (one SM, and SM pairs) load a group's last k-block
+with a 16-, 32- or 48-row box.  Here every group of one launch has its own
+load, covering each residue (0, 1, 15-17, 31-33, ..., 127, 128 rows of a
+128-row capacity; up to 256 rows of a 256-row one), and every
 padding row of the inputs (rows s >= load of xe, dye and the workspace) holds
 NaN: padding contents must not reach any output.  The forward outputs' padding
 rows must keep what the caller left there (they are not written).  The bf16
@@ -21,7 +22,11 @@ from gpu_helpers import np64, rel_err, rms_err
 pytestmark = pytest.mark.gpu
 
 LOADS = [0, 1, 15, 16, 17, 31, 32, 33, 47, 48, 49, 63, 64, 65, 79, 80, 96, 111, 112, 113, 127, 128]
-C = 128
+# capacity 256: every residue of the last of up to four k-blocks
+LOADS_256 = [0, 1, 16, 33, 64, 65, 100, 127, 128, 129, 143, 160, 191, 192, 193, 209, 224, 239, 255, 256]
+# capacity 32 (the SM-pair kernel for dW2 too): one partial k-block per group
+LOADS_32 = [0, 1, 2, 7, 8, 15, 16, 17, 24, 31, 32, 0, 5]
+LOADS_BY_C = {32: LOADS_32, 128: LOADS, 256: LOADS_256}
 SENTINEL = 7.0
 
 
@@ -31,11 +36,11 @@ def _lib():
     __graft_entry__.build()
 
 
-def _inputs(dtype, d, f, seed=90):
+def _inputs(dtype, d, f, loads, C, seed=90):
     g = torch.Generator().manual_seed(seed)
-    G = len(LOADS)
+    G = len(loads)
     tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
-    load = torch.tensor(LOADS, dtype=torch.int32).reshape(1, G)
+    load = torch.tensor(loads, dtype=torch.int32).reshape(1, G)
     valid = torch.arange(C)[None, :] < load.reshape(G, 1)  # [G, C]
 
     def rows(width, scale):
@@ -56,13 +61,23 @@ def _zero_pad(t, valid):
     return t
 
 
-@pytest.mark.parametrize("dtype,d,f", [("bf16", 128, 256), ("bf16", 256, 384), ("f32", 40, 72)])
-def test_group_tails(dtype, d, f):
+# d 128 / f 256 and d 256 / f 384: the one-SM weight-gradient kernels (resident B,
+# and streaming with 128-column tiles); d 256 / f 512 and d 512 / f 256: the
+# SM-pair kernel for dW1 (C 128: two resident B tiles; C 256: one) and for dW2
+# (C 32 and C 256; with C 128 dW2 streams).  With C 256 the row-mode GEMMs run on
+# SM pairs (256-row tiles), with 256-column tiles (d 512 / f 256) and 128-column
+# ones (d 384 / f 640, whose weight gradients stream).
+@pytest.mark.parametrize("dtype,d,f,C", [("bf16", 128, 256, 128), ("bf16", 256, 384, 128),
+                                         ("bf16", 256, 512, 128), ("bf16", 512, 256, 256),
+                                         ("bf16", 256, 512, 32), ("bf16", 384, 640, 256),
+                                         ("f32", 40, 72, 128)])
+def test_group_tails(dtype, d, f, C):
     import paper_2608_16188_gb300 as vm
-    G = len(LOADS)
+    loads = LOADS_BY_C[C]
+    G = len(loads)
     p = vm.problem(1, C, d, f, G, 1, 1.0, dtype, capacity=C)
     assert vm.vmoe_problem_capacity(p) == C
-    load, valid, xe, dye, w1, w2 = _inputs(dtype, d, f)
+    load, valid, xe, dye, w1, w2 = _inputs(dtype, d, f, loads, C)
     dev = "cuda"
     tdt = xe.dtype
     xe_d, dye_d, w1_d, w2_d, load_d = (t.to(dev) for t in (xe, dye, w1, w2, load))
@@ -79,7 +94,7 @@ def test_group_tails(dtype, d, f):
 
     tol, agg = (2e-2, 5e-3) if dtype == "bf16" else (1e-5, 2.5e-6)
     xe0, dye0 = _zero_pad(xe, valid), _zero_pad(dye, valid)
-    r_h, r_a, r_ye = oracle.expert_fwd(xe0, np64(w1), np64(w2), LOADS)
+    r_h, r_a, r_ye = oracle.expert_fwd(xe0, np64(w1), np64(w2), loads)
     for name, gpu, ref in (("h", h, r_h), ("a", a, r_a), ("ye", ye, r_ye)):
         g64 = np64(gpu)
         assert np.all(np.isfinite(g64[vmask])), name
@@ -90,7 +105,7 @@ def test_group_tails(dtype, d, f):
     # backward: the oracle takes the forward outputs this call received
     h_in = _zero_pad(h.cpu(), valid)
     a_in = _zero_pad(a.cpu(), valid)
-    _, r_dxe, r_dw1, r_dw2 = oracle.expert_bwd(xe0, h_in, a_in, np64(w1), np64(w2), dye0, LOADS)
+    _, r_dxe, r_dw1, r_dw2 = oracle.expert_bwd(xe0, h_in, a_in, np64(w1), np64(w2), dye0, loads)
     full = vm.vmoe_expert_bwd_workspace_size(p)
     sizes = [full] + ([vm.vmoe_expert_bwd_min_workspace_size(p)] if dtype == "bf16" else [])
     results = []
@@ -116,3 +131,21 @@ def test_group_tails(dtype, d, f):
     if len(results) == 2:  # the sliced run is bitwise the full one
         for x, y in zip(results[0], results[1]):
             assert torch.equal(x, y)
+
+
+# The row-mode SM-pair kernel (256-row tiles) is off by default and switched on by
+# VMOE_ROW_PAIR=1, which the library reads once per process: the capacity-256
+# cases run again in a child process with it set.
+@pytest.mark.parametrize("d,f", [(512, 256), (384, 640)])
+def test_group_tails_row_pair(d, f):
+    import os
+    import subprocess
+    import sys
+    here = os.path.dirname(os.path.abspath(__file__))
+    code = ("import sys; sys.path[:0] = [%r, %r]; import test_gpu_tails as t; "
+            "t.test_group_tails('bf16', %d, %d, 256); print('ROW_PAIR_OK')"
+            % (here, os.path.dirname(here), d, f))
+    env = dict(os.environ, VMOE_ROW_PAIR="1")
+    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                       timeout=600)
+    assert r.returncode == 0 and "ROW_PAIR_OK" in r.stdout, r.stdout[-2000:] + r.stderr[-2000:]
