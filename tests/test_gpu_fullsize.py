@@ -17,7 +17,7 @@ import torch
 
 import oracle
 import workloads
-from gpu_helpers import (BF16_RMS_TOL, BF16_TOL, np64, rel_err, rms_err, run_step, to_dev,
+from gpu_helpers import (BF16_RMS_TOL, BF16_TOL, np64, rel_err, report, run_step, to_dev,
                          valid_rows)
 
 pytestmark = pytest.mark.gpu
@@ -29,8 +29,8 @@ def _lib():
     __graft_entry__.build()
 
 
-def _ok(name, g, r, mask=None, errs=None, groups=None):
-    e = (rel_err(g, r, mask, groups), rms_err(g, r, mask, groups))
+def _ok(name, g, r, mask=None, errs=None, groups=None, case="fullsize"):
+    e = report(case, name, g, r, mask, groups)
     if errs is not None:
         errs[name] = e
     return e[0] <= BF16_TOL and e[1] <= BF16_RMS_TOL
@@ -65,13 +65,13 @@ def test_fullsize_sampled_parity(name):
         assert np.array_equal(np64(b.xe[t:t + 1]), xe_ref)
         dye_ref = oracle.dispatch(inp["dy"][t:t + 1], rgate[t:t + 1], ridx[t:t + 1],
                                   rslot[t:t + 1], E, C)
-        assert _ok("dye", b.dye[t:t + 1], dye_ref, errs=errs, groups=E), errs
+        assert _ok("dye", b.dye[t:t + 1], dye_ref, errs=errs, groups=E, case=name), errs
 
     # combine at full size from the GPU's own expert outputs
     y_ref = oracle.combine(b.ye, rgate, ridx, rslot, N)
-    assert _ok("y", b.y, y_ref, errs=errs, groups=T * N), errs
+    assert _ok("y", b.y, y_ref, errs=errs, groups=T * N, case=name), errs
     dx_ref = oracle.combine(b.dxe, None, ridx, rslot, N)
-    assert _ok("dx", b.dx, dx_ref, errs=errs, groups=T * N), errs
+    assert _ok("dx", b.dx, dx_ref, errs=errs, groups=T * N, case=name), errs
 
     # sampled groups through the whole expert FFN, forward and backward
     G = T * E
@@ -99,7 +99,7 @@ def test_fullsize_sampled_parity(name):
               ("dw1", b.dw1.view(G, cfg.d, cfg.f)[picks], dw1, None),
               ("dw2", b.dw2.view(G, cfg.f, cfg.d)[picks], dw2, None)]
     ng = len(picks)
-    bad = [nm for nm, g_, r_, m_ in checks if not _ok(nm, g_, r_, m_, errs, groups=ng)]
+    bad = [nm for nm, g_, r_, m_ in checks if not _ok(nm, g_, r_, m_, errs, groups=ng, case=name)]
     assert not bad, (name, picks, ld.tolist(), errs)
     if empty.size:
         e0 = int(empty[0])

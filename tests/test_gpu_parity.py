@@ -16,7 +16,7 @@ import torch
 import oracle
 import workloads
 from gpu_helpers import (BF16_RMS_TOL, BF16_TOL, F32_RMS_TOL, F32_TOL, GATE_RTOL, np64, problem_of,
-                         rel_err, rms_err, run_step, to_dev, valid_rows)
+                         rel_err, report, rms_err, run_step, to_dev, valid_rows)
 
 pytestmark = pytest.mark.gpu
 
@@ -38,6 +38,13 @@ SMALL = {
     "bf16_norenorm_tanh": Config("bf16_norenorm_tanh", 23, T=2, N=160, d=128, f=384, E=4, k=2,
                                  cf=1.5, dtype="bf16", flags=2 | 4),
 }
+
+
+# Cases whose end-to-end dW1 / dW2 meet the per-element bar (measured: 0.007-0.019);
+# the others (bf16_bn128_drops, capacity_one, k8_of_256_experts) sit at 0.021-0.031,
+# the floor that bf16 A and dYe set, and are held to the aggregate bar.
+E2E_DW_ELEMENTWISE = {"bf16_two_mtiles", "bf16_skew_empty", "bf16_norenorm_tanh", "k_equals_E",
+                      "one_token", "1024_groups"}
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -81,10 +88,17 @@ def _compare_step(cfg, inp_cpu, b, flags):
         "dw2": (b.dw2, s_dw2, None, G), "dx_stage": (b.dx, s_dx, None, T * N),
         "y_e2e": (b.y, ref["y"], None, T * N), "dx_e2e": (b.dx, ref["dx"], None, T * N),
     }
-    errs = {n: (rel_err(g, r, m, gr), rms_err(g, r, m, gr)) for n, (g, r, m, gr) in checks.items()}
-    # end-to-end weight gradients: aggregate bar (their inputs A and dYe are bf16 by the ABI)
-    errs["dw1_e2e_rms"] = (0.0, rms_err(b.dw1, ref["dw1"]))
-    errs["dw2_e2e_rms"] = (0.0, rms_err(b.dw2, ref["dw2"]))
+    errs = {n: report(cfg.name, n, g, r, m, gr) for n, (g, r, m, gr) in checks.items()}
+    # end-to-end weight gradients: their inputs A and dYe are bf16 by the ABI, and a
+    # CPU emulation of exactly those roundings reaches 0.021-0.031 per element on the
+    # cases with the fewest rows per group and the largest cancellation; those are held
+    # to the aggregate bar, every other case also to the per-element one
+    e_dw1 = report(cfg.name, "dw1_e2e", b.dw1, ref["dw1"], None, G)
+    e_dw2 = report(cfg.name, "dw2_e2e", b.dw2, ref["dw2"], None, G)
+    if cfg.name in E2E_DW_ELEMENTWISE or cfg.dtype == "f32":
+        errs["dw1_e2e"], errs["dw2_e2e"] = e_dw1, e_dw2
+    else:
+        errs["dw1_e2e_rms"], errs["dw2_e2e_rms"] = (0.0, e_dw1[1]), (0.0, e_dw2[1])
     bad = {n: v for n, v in errs.items() if not (v[0] <= tol and v[1] <= rms_tol)}
     print(cfg.name, {n: (round(v[0], 5), round(v[1], 6)) for n, v in errs.items()})
     assert not bad, (cfg.name, bad)
