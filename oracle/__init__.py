@@ -22,6 +22,10 @@ Parity status (what pins each function, see ``tests/test_oracle_pins.py``):
                   gates differentiable) and central finite differences
   plan_slices     (planner.py, plain Python) brute-force subset enumeration, a
                   textbook knapsack instance, equal-weight closed forms
+  fill_clamp_refill / integer_shares  (planner.py) the closed form
+                  min(sat, min + lambda w) with lambda found by bisection, a
+                  hand-worked example (tests/golden/shares_example.json), sums
+                  and bounds, rounding within one unit
 """
 from __future__ import annotations
 
@@ -33,6 +37,7 @@ import threading
 import numpy as np
 
 from .planner import plan_slices  # noqa: F401  (cross-task slice planner, Section 3.2.1)
+from .planner import fill_clamp_refill, integer_shares  # noqa: F401  (Section 3.2.2)
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "vmoe_oracle.c")

@@ -89,3 +89,63 @@ def plan_slices(weight, lifespan, capacity: int, eta: float = 0.0, budget: float
 def slice_value(slice_items, weight, lifespan, capacity, eta=0.0, budget=None):
     mc = float(capacity if budget is None else budget)
     return sum((weight[i] / mc if mc > 0 else 0.0) - eta * lifespan[i] for i in slice_items)
+
+
+def fill_clamp_refill(work, minimum, saturation, budget):
+    """Resource shares of co-running experts (Section 3.2.2, lifespan-aware
+    aligning): the controller's fill-clamp-refill allocation, real-valued.
+
+      1. seed: every expert gets its minimum;
+      2. fill: the budget left is shared out in proportion to the work
+         coefficients of the experts not yet saturated;
+      3. clamp: an expert above its saturation point is cut back to it, and what
+         it gave up is shared out again over the others (step 2), until nothing
+         is left or every expert with work is saturated.
+
+    Readings (the paper gives the three steps, not their arithmetic):
+      * an expert with no work (coefficient 0) keeps its minimum;
+      * an expert whose share reaches its saturation exactly counts as clamped;
+      * a budget below the sum of the minima is an error;
+      * what is left when every expert with work is saturated stays unallocated.
+    float64 throughout, sums in index order.  Returns (shares, unallocated)."""
+    n = len(work)
+    w = [float(x) for x in work]
+    sat = [float(x) for x in saturation]
+    a = [float(x) for x in minimum]
+    if any(x < 0 for x in w) or any(a[i] < 0 or sat[i] < a[i] for i in range(n)):
+        raise ValueError("negative work or minimum, or saturation below minimum")
+    left = float(budget) - sum(a)
+    if left < 0:
+        raise ValueError("the minima exceed the budget")
+    active = [i for i in range(n) if w[i] > 0 and a[i] < sat[i]]
+    while left > 0 and active:
+        wsum = 0.0
+        for i in active:
+            wsum += w[i]
+        for i in active:
+            a[i] += left * w[i] / wsum
+        left = 0.0
+        still = []
+        for i in active:
+            if a[i] >= sat[i]:
+                left += a[i] - sat[i]
+                a[i] = sat[i]
+            else:
+                still.append(i)
+        active = still
+    return a, left
+
+
+def integer_shares(work, minimum, saturation, budget):
+    """fill_clamp_refill rounded to whole units (CTAs): every share is floored,
+    then the units still missing from the real-valued total go one each to the
+    largest fractional parts (ties to the lower index).  A real share lies in
+    [minimum, saturation], both integers, so the rounded one does too."""
+    x, _ = fill_clamp_refill(work, minimum, saturation, budget)
+    fl = [int(np.floor(v)) for v in x]
+    total = int(round(sum(x)))
+    missing = total - sum(fl)
+    frac = sorted(range(len(x)), key=lambda i: (-(x[i] - fl[i]), i))
+    for i in frac[:missing]:
+        fl[i] += 1
+    return fl
