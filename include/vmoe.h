@@ -270,6 +270,24 @@ int vmoe_router_bwd(const vmoe_problem *p, const void *x, const float *w_router,
 int vmoe_plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity,
                      double eta, double budget, int32_t *order, int32_t *slice_start);
 
+/* Resource shares of co-running experts (Section 3.2.2, lifespan-aware
+ * aligning; host code, no GPU): the fill-clamp-refill allocation of `budget`
+ * units among n experts -- each is seeded with minimum[i]; what is left is
+ * shared out in proportion to work[i] among the experts below their
+ * saturation[i]; an expert above its saturation is clamped to it and what it
+ * gave up is shared out again, until nothing is left or every expert with work
+ * is saturated.  An expert with work 0 keeps its minimum.  The real-valued
+ * shares are then rounded to whole units: floored, and the units still
+ * missing from their total given one each to the largest fractional parts
+ * (ties to the lower index), so minimum[i] <= shares[i] <= saturation[i].
+ * float64 arithmetic, sums in index order.
+ * Output: shares[n].  Returns the number of units allocated (budget, or less
+ * when the saturations do not reach it), VMOE_ERR_INVALID (null pointers,
+ * negative or NaN work, negative minimum, saturation below minimum) or
+ * VMOE_ERR_UNSUPPORTED (the minima exceed the budget). */
+int vmoe_plan_shares(int n, const double *work, const int32_t *minimum, const int32_t *saturation,
+                     int32_t budget, int32_t *shares);
+
 /* Device status word of the current device: 0 when clean, otherwise a
  * vmoe_status (VMOE_ERR_DEVICE_TIMEOUT after a kernel gave up a bounded
  * wait).  Synchronises the current device.  `reset` != 0 clears the word. */

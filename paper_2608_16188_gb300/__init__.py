@@ -35,7 +35,7 @@ VMOE_GELU_TANH = 1 << 2
 EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_route",
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
            "vmoe_expert_bwd_min_workspace_size",
-           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd", "vmoe_plan_slices",
+           "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd", "vmoe_plan_slices", "vmoe_plan_shares",
            "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
            "vmoe_trace_disable", "vmoe_trace_get")
 
@@ -83,6 +83,7 @@ def library():
             "vmoe_router_bwd": (ctypes.c_int, [PP] + [_P] * 13 + [_P]),
             "vmoe_plan_slices": (ctypes.c_int, [ctypes.c_int, _P, _P, ctypes.c_int64,
                                                 ctypes.c_double, ctypes.c_double, _P, _P]),
+            "vmoe_plan_shares": (ctypes.c_int, [ctypes.c_int, _P, _P, _P, ctypes.c_int32, _P]),
             "vmoe_device_status": (ctypes.c_int, [ctypes.c_int]),
             "vmoe_selftest_bounded_wait": (ctypes.c_int, [ctypes.c_longlong, _P]),
             "vmoe_trace_enable": (ctypes.c_int, [ctypes.c_int]),
@@ -220,6 +221,21 @@ def vmoe_plan_slices(weight, lifespan, capacity: int, eta: float = 0.0, budget: 
                                     float(budget), order.ctypes.data, start.ctypes.data)
     _check(ns if ns < 0 else 0, "vmoe_plan_slices")
     return [order[start[s]:start[s + 1]].tolist() for s in range(ns)]
+
+
+def vmoe_plan_shares(work, minimum, saturation, budget: int):
+    """Host-side fill-clamp-refill allocation (see include/vmoe.h); returns the
+    list of whole-unit shares."""
+    import numpy as np
+    w = np.ascontiguousarray(work, dtype=np.float64)
+    mn = np.ascontiguousarray(minimum, dtype=np.int32)
+    sat = np.ascontiguousarray(saturation, dtype=np.int32)
+    n = int(w.size)
+    out = np.zeros(max(n, 1), dtype=np.int32)
+    r = library().vmoe_plan_shares(n, w.ctypes.data, mn.ctypes.data, sat.ctypes.data, int(budget),
+                                   out.ctypes.data)
+    _check(r if r < 0 else 0, "vmoe_plan_shares")
+    return out[:n].tolist()
 
 
 def vmoe_device_status(reset: bool = False) -> int:

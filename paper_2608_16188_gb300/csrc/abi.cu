@@ -45,6 +45,14 @@ bool pair_enabled() {
     return on;
 }
 
+bool shares_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("VMOE_SHARES");
+        return v && v[0] == '1';
+    }();
+    return on;
+}
+
 bool row_pair_enabled() {
     static const bool on = [] {
         const char *v = getenv("VMOE_ROW_PAIR");

@@ -49,6 +49,9 @@ bool pdl_enabled();  // abi.cu
 // groups above 128 rows, off unless VMOE_ROW_PAIR=1.
 bool pair_enabled();
 bool row_pair_enabled();
+// The fill-clamp-refill pair shares of the memory-budgeted backward's dW1,
+// off unless VMOE_SHARES=1 (abi.cu).
+bool shares_enabled();
 
 template <typename... KArgs, typename... Args>
 int launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,

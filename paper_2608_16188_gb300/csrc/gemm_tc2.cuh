@@ -172,6 +172,20 @@ struct PairShape {
     static_assert(SMEM_BYTES <= 232448, "over the 227 KB shared-memory limit");
 };
 
+// Which units each SM pair works on.  By default (enabled = 0) pair c takes
+// units c, c + P, c + 2P, ... of P pairs -- a static round-robin over units
+// of nearly equal cost.  With enabled = 1 pair c takes the contiguous units
+// [first[c], first[c] + count[c]): the per-group pair shares of the
+// fill-clamp-refill allocation (Section 3.2.2), each group's units split
+// evenly over the pairs of its share (vmoe_plan_shares; the memory-budgeted
+// backward, whose loads are on the host).
+constexpr int MAX_PAIRS = 128;
+struct PairSchedule {
+    int enabled;
+    int32_t first[MAX_PAIRS];
+    int32_t count[MAX_PAIRS];
+};
+
 // K rows of a group with load L are taken in nkb = ceil(L / 64) k-blocks
 // aligned to the END of its rows: k-block j covers rows [L - 64 (nkb - j),
 // L - 64 (nkb - j - 1)), so only k-block 0 is partial and its missing rows lie
@@ -184,7 +198,7 @@ template <bool KSPLIT, int NKB>
 __global__ void __launch_bounds__(THREADS, 1)
 wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                   const __grid_constant__ CUtensorMap tmBlo, const __grid_constant__ CUtensorMap tmD,
-                  Args args) {
+                  Args args, const __grid_constant__ PairSchedule sched) {
     using S = PairShape<KSPLIT, NKB>;
     constexpr uint32_t IDESC = idesc_bf16(S::MP, S::BN, true, true);
     constexpr int AS = S::A_SLOTS, BB = S::B_BUFS;
@@ -249,6 +263,10 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     const int total = args.G * args.tiles_n;
     const int tiles_m = args.tiles_m;  // M / 256
     const bool cmpb = (args.compact & CMP_B) != 0;  // B rows from crow, residual after L
+    // this pair's units: u = u_first, u_first + u_step, ... < u_end
+    const int u_first = sched.enabled ? sched.first[cid] : cid;
+    const int u_step = sched.enabled ? 1 : ncl;
+    const int u_end = sched.enabled ? min(total, sched.first[cid] + sched.count[cid]) : total;
     int crow = 0;
     auto decode = [&](int u, int &g, int &n_blk, int &L) {
         const int i = u / args.tiles_n;
@@ -268,10 +286,10 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             int ub = 0, ka = 0;
             bool ok = true;
             int b_issued[BB] = {}, a_issued[AS] = {};
-            for (int u = cid; u < total && ok; u += ncl) {
+            for (int u = u_first; u < u_end && ok; u += u_step) {
                 int g, n_blk, L;
                 decode(u, g, n_blk, L);
-                if (u + ncl >= total) pdl_launch_dependents();  // this pair's last unit
+                if (u + u_step >= u_end) pdl_launch_dependents();  // this pair's last unit
                 const int nkb = (L + BK - 1) / BK;
                 if (nkb == 0) continue;
                 const int r0 = L - nkb * BK;  // first row of k-block 0 (<= 0)
@@ -332,7 +350,7 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         // ------------------------------------------------------------ B hand-over (+ MMA in the leader)
         int ub = 0, ka = 0, it = 0;
         bool ok = true;
-        for (int u = cid; u < total && ok; u += ncl) {
+        for (int u = u_first; u < u_end && ok; u += u_step) {
             int g, n_blk, L;
             decode(u, g, n_blk, L);
             const int nkb = (L + BK - 1) / BK;
@@ -418,7 +436,7 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         uint8_t *stg = epi_base + ew * S::STG_BUFS * 4096;
         int nstore = 0, it = 0;
         bool ok = true;
-        for (int u = cid; u < total && ok; u += ncl) {
+        for (int u = u_first; u < u_end && ok; u += u_step) {
             int g, n_blk, L;
             decode(u, g, n_blk, L);
             for (int m = 0; m < tiles_m; ++m) {
@@ -913,7 +931,8 @@ int pair_clusters(const void *kern, size_t smem);
 
 template <bool KSPLIT, int NKB>
 int launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mblo, const CUtensorMap &md,
-                const Args &a, long long units, cudaStream_t s, const char *name) {
+                const Args &a, long long units, cudaStream_t s, const char *name,
+                const PairSchedule *sched = nullptr) {
     using S = PairShape<KSPLIT, NKB>;
     auto kern = wgrad_pair_kernel<KSPLIT, NKB>;
     static std::atomic<int> smem_limit[64];
@@ -921,7 +940,18 @@ int launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap 
     if (units <= 0) return VMOE_OK;
     const int ncl = pair_clusters((const void *)kern, S::SMEM_BYTES);
     if (ncl <= 0) return VMOE_ERR_CUDA;
-    const long long clusters = units < ncl ? units : ncl;
+    long long clusters = units < ncl ? units : ncl;
+    PairSchedule sc;
+    sc.enabled = 0;
+    if (sched && sched->enabled) {  // a share schedule names its own pairs
+        sc = *sched;
+        int used = 0;
+        for (int c = 0; c < MAX_PAIRS; ++c)
+            if (sc.count[c] > 0) used = c + 1;
+        if (used > ncl) return VMOE_ERR_INVALID;
+        clusters = used;
+    }
+    if (clusters <= 0) return VMOE_OK;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(2 * clusters));
     cfg.blockDim = dim3(THREADS);
@@ -937,7 +967,7 @@ int launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap 
     cfg.attrs = attr;
     cfg.numAttrs = pdl_enabled() ? 2 : 1;
     trace_before(s, name);
-    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, ma, mb, mblo, md, a);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, ma, mb, mblo, md, a, sc);
     trace_after(s);
     return e == cudaSuccess ? VMOE_OK : VMOE_ERR_CUDA;
 }
@@ -972,6 +1002,22 @@ int launch_row_pair(const CUtensorMap &ma, const CUtensorMap &mb, const TailMaps
     const cudaError_t e = cudaLaunchKernelEx(&cfg, kern, ma, mb, mat, a);
     trace_after(s);
     return e == cudaSuccess ? VMOE_OK : VMOE_ERR_CUDA;
+}
+
+// SM pairs the weight-gradient kernel for capacity C runs on at once (its
+// dynamic shared-memory limit raised first); 0 if the query fails.
+template <bool KSPLIT>
+int pair_wgrad_capacity(int C) {
+    if (C <= 2 * BK) {
+        using S = PairShape<KSPLIT, 2>;
+        static std::atomic<int> lim[64];
+        if (raise_smem_limit((const void *)wgrad_pair_kernel<KSPLIT, 2>, lim, (int)S::SMEM_BYTES)) return 0;
+        return pair_clusters((const void *)wgrad_pair_kernel<KSPLIT, 2>, S::SMEM_BYTES);
+    }
+    using S = PairShape<KSPLIT, 4>;
+    static std::atomic<int> lim[64];
+    if (raise_smem_limit((const void *)wgrad_pair_kernel<KSPLIT, 4>, lim, (int)S::SMEM_BYTES)) return 0;
+    return pair_clusters((const void *)wgrad_pair_kernel<KSPLIT, 4>, S::SMEM_BYTES);
 }
 
 // Row-mode GEMM: D[g][C rows][N] = act[g][C][K] * B, B MN-major ([K][N]) or
@@ -1048,7 +1094,8 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
 // VMOE_PAIR=0 in the environment turns the pair kernel off.
 inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __nv_bfloat16 *act2,
                       int N, const int32_t *load, __nv_bfloat16 *D, cudaStream_t s,
-                      const char *name, bool ksplit = false, const Slice &sl = Slice()) {
+                      const char *name, bool ksplit = false, const Slice &sl = Slice(),
+                      const PairSchedule *sched = nullptr) {
     const int G = p.G(), C = p.C;
     const bool wide = N % 256 == 0;
     const int BN = wide ? 256 : 128;
@@ -1099,10 +1146,10 @@ inline int wgrad_gemm(const Dims &p, const __nv_bfloat16 *act1, int M, const __n
         a.tiles_n = N / 256;
         const long long units = (long long)a.G * a.tiles_n;
         if (C <= 2 * BK)
-            return ksplit ? launch_pair<true, 2>(ma, mb, mblo, md, a, units, s, name)
-                          : launch_pair<false, 2>(ma, mb, mblo, md, a, units, s, name);
-        return ksplit ? launch_pair<true, 4>(ma, mb, mblo, md, a, units, s, name)
-                      : launch_pair<false, 4>(ma, mb, mblo, md, a, units, s, name);
+            return ksplit ? launch_pair<true, 2>(ma, mb, mblo, md, a, units, s, name, sched)
+                          : launch_pair<false, 2>(ma, mb, mblo, md, a, units, s, name, sched);
+        return ksplit ? launch_pair<true, 4>(ma, mb, mblo, md, a, units, s, name, sched)
+                      : launch_pair<false, 4>(ma, mb, mblo, md, a, units, s, name, sched);
     }
     if (!make_map_chunked(&ma, act1, M, C, G, 64, BM / 64)) return VMOE_ERR_CUDA;
     if (!make_map_chunked(&mb, act2, N, b_rows, b_outer, 64, BN / 64)) return VMOE_ERR_CUDA;

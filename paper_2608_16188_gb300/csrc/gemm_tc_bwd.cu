@@ -11,6 +11,8 @@ namespace vmoe {
 
 int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
                 double budget, int32_t *order, int32_t *slice_start);  // planner.cu
+int plan_shares(int n, const double *work, const int32_t *minimum, const int32_t *saturation,
+                int32_t budget, int32_t *shares);                      // planner.cu
 
 namespace tc {
 int pair_clusters(const void *kern, size_t smem) {
@@ -140,6 +142,36 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
         cudaSuccess)
         return VMOE_ERR_CUDA;
     if (cudaStreamSynchronize(s) != cudaSuccess) return VMOE_ERR_CUDA;  // host plan buffer is freed on return
+    // dW1 of a slice on SM pairs, optionally (VMOE_SHARES=1) with each group's
+    // column tiles on a share of the pairs from the fill-clamp-refill allocation
+    // (Section 3.2.2): work = its tiles x (output bytes + load x input bytes per
+    // row), at least one pair, at most one pair per tile; slices with more
+    // groups than pairs keep the round-robin schedule.
+    const bool use_shares = shares_enabled() && pair_enabled() && p.d % 256 == 0 && p.f % 256 == 0 &&
+                            p.C <= 4 * BK;
+    const int pairs = use_shares ? pair_wgrad_capacity<true>(p.C) : 0;
+    auto slice_schedule = [&](int sidx, PairSchedule &sc) {
+        sc.enabled = 0;
+        const int n = start[sidx + 1] - start[sidx];
+        if (pairs <= 0 || n > pairs || pairs > MAX_PAIRS) return;
+        const int units = p.f / 256, tiles_m = p.d / 256;
+        std::vector<double> work(n);
+        std::vector<int32_t> mn(n, 1), sat(n, units), share(n);
+        for (int i = 0; i < n; ++i) {
+            const double L = hload[order[start[sidx] + i]];
+            work[i] = units * ((double)tiles_m * 256 * 256 * 2 + L * ((double)p.d * 2 + 4 * 256));
+        }
+        if (plan_shares(n, work.data(), mn.data(), sat.data(), pairs, share.data()) < 0) return;
+        int c = 0;
+        for (int i = 0; i < n; ++i)
+            for (int j = 0; j < share[i]; ++j, ++c) {
+                const int lo = j * units / share[i], hi = (j + 1) * units / share[i];
+                sc.first[c] = i * units + lo;
+                sc.count[c] = hi - lo;
+            }
+        for (; c < MAX_PAIRS; ++c) sc.first[c] = sc.count[c] = 0;
+        sc.enabled = 1;
+    };
     int st = VMOE_OK;
     for (int sidx = 0; sidx < ns && st == VMOE_OK; ++sidx) {
         Slice sl;
@@ -156,7 +188,9 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
                                         0, 0, sl);
         if (st != VMOE_OK) break;
         sl.compact = CMP_B;
-        st = wgrad_gemm(p, xe, p.d, dh, p.f, load, dw1, s, "tc_dw1", true, sl);
+        PairSchedule sc;
+        slice_schedule(sidx, sc);
+        st = wgrad_gemm(p, xe, p.d, dh, p.f, load, dw1, s, "tc_dw1", true, sl, &sc);
     }
     if (st == VMOE_OK) st = wgrad_gemm(p, act, p.f, dye, p.d, load, dw2, s, "tc_dw2");
     if (nslices_out) *nslices_out = ns;

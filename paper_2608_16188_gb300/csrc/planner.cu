@@ -15,6 +15,8 @@
 // slice; an expert heavier than the budget is refused.
 #include <stdint.h>
 
+#include <math.h>
+
 #include <algorithm>
 #include <memory>
 #include <numeric>
@@ -100,7 +102,71 @@ int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t ca
     return (int)slices.size();
 }
 
+// Section 3.2.2 (lifespan-aware aligning): the fill-clamp-refill allocation of a
+// budget of resources among co-running experts -- seed each with its minimum,
+// share the rest out in proportion to the work coefficients of the experts not
+// yet saturated, clamp those above their saturation and share out again what
+// they gave up -- then rounded to whole units: shares floored, the units still
+// missing from the real-valued total to the largest fractional parts (ties to
+// the lower index).  Readings: an expert with no work keeps its minimum; one
+// that reaches its saturation exactly counts as clamped; what is left once
+// every expert with work is saturated stays unallocated.  float64, sums in
+// index order.  Returns the number of units allocated.
+int plan_shares(int n, const double *work, const int32_t *minimum, const int32_t *saturation,
+                int32_t budget, int32_t *shares) {
+    if (n < 0 || budget < 0 || (n > 0 && (!work || !minimum || !saturation || !shares)))
+        return VMOE_ERR_INVALID;
+    std::vector<double> a(n);
+    double msum = 0.0;
+    for (int i = 0; i < n; ++i) {
+        if (!(work[i] >= 0.0) || minimum[i] < 0 || saturation[i] < minimum[i]) return VMOE_ERR_INVALID;
+        a[i] = (double)minimum[i];
+        msum += a[i];
+    }
+    double left = (double)budget - msum;
+    if (left < 0.0) return VMOE_ERR_UNSUPPORTED;  // the minima exceed the budget
+    std::vector<int> active, still;
+    for (int i = 0; i < n; ++i)
+        if (work[i] > 0.0 && a[i] < (double)saturation[i]) active.push_back(i);
+    while (left > 0.0 && !active.empty()) {
+        double wsum = 0.0;
+        for (int i : active) wsum += work[i];
+        for (int i : active) a[i] += left * work[i] / wsum;
+        left = 0.0;
+        still.clear();
+        for (int i : active) {
+            const double s = (double)saturation[i];
+            if (a[i] >= s) {
+                left += a[i] - s;
+                a[i] = s;
+            } else {
+                still.push_back(i);
+            }
+        }
+        active.swap(still);
+    }
+    double xsum = 0.0;
+    int64_t fsum = 0;
+    std::vector<int> idx(n);
+    for (int i = 0; i < n; ++i) {
+        xsum += a[i];
+        shares[i] = (int32_t)std::floor(a[i]);
+        fsum += shares[i];
+        idx[i] = i;
+    }
+    const int64_t total = std::llround(xsum);
+    std::stable_sort(idx.begin(), idx.end(),
+                     [&](int p, int q) { return a[p] - shares[p] > a[q] - shares[q]; });
+    for (int64_t r = 0; r < total - fsum && r < n; ++r) shares[idx[r]] += 1;
+    return (int)total;
+}
+
 }  // namespace vmoe
+
+extern "C" int vmoe_plan_shares(int n, const double *work, const int32_t *minimum,
+                                const int32_t *saturation, int32_t budget, int32_t *shares) {
+    return vmoe::plan_shares(n, work, minimum, saturation, budget, shares);
+}
 
 extern "C" int vmoe_plan_slices(int n, const int64_t *weight, const double *lifespan,
                                 int64_t capacity, double eta, double budget, int32_t *order,

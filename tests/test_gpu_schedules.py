@@ -1,0 +1,48 @@
+"""The library's optional schedules, each switched on by an environment variable
+that it reads once per process, run the GPU parity tests again in a child process:
+
+  VMOE_ROW_PAIR=1  row-mode GEMMs of groups above 128 rows on SM pairs (256-row
+                   tiles): the capacity-256 group-tail cases, against the oracle
+                   and sliced against full, bitwise;
+  VMOE_SHARES=1    the memory-budgeted backward's dW1 with each group's column
+                   tiles on a share of the SM pairs from the fill-clamp-refill
+                   allocation (Section 3.2.2): the sliced-backward cases, which
+                   must stay bitwise equal to the unsliced backward, and the
+                   group-tail cases.
+"""
+import os
+import subprocess
+import sys
+
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    import __graft_entry__
+    __graft_entry__.build()
+
+
+def _child(env_name, targets):
+    env = dict(os.environ, **{env_name: "1"})
+    r = subprocess.run([sys.executable, "-m", "pytest", "-q", "-x", "-p", "no:cacheprovider", *targets],
+                       cwd=os.path.dirname(HERE), env=env, capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stdout[-3000:] + r.stderr[-2000:]
+    return r.stdout
+
+
+def test_row_pair_schedule():
+    out = _child("VMOE_ROW_PAIR", ["tests/test_gpu_tails.py::test_group_tails[bf16-512-256-256]",
+                                   "tests/test_gpu_tails.py::test_group_tails[bf16-384-640-256]"])
+    assert "2 passed" in out
+
+
+def test_share_schedule():
+    out = _child("VMOE_SHARES", ["tests/test_gpu_sliced_bwd.py",
+                                 "tests/test_gpu_tails.py::test_group_tails[bf16-256-512-128]",
+                                 "tests/test_gpu_tails.py::test_group_tails[bf16-512-256-256]"])
+    assert "passed" in out and "failed" not in out

@@ -132,20 +132,3 @@ def test_group_tails(dtype, d, f, C):
         for x, y in zip(results[0], results[1]):
             assert torch.equal(x, y)
 
-
-# The row-mode SM-pair kernel (256-row tiles) is off by default and switched on by
-# VMOE_ROW_PAIR=1, which the library reads once per process: the capacity-256
-# cases run again in a child process with it set.
-@pytest.mark.parametrize("d,f", [(512, 256), (384, 640)])
-def test_group_tails_row_pair(d, f):
-    import os
-    import subprocess
-    import sys
-    here = os.path.dirname(os.path.abspath(__file__))
-    code = ("import sys; sys.path[:0] = [%r, %r]; import test_gpu_tails as t; "
-            "t.test_group_tails('bf16', %d, %d, 256); print('ROW_PAIR_OK')"
-            % (here, os.path.dirname(here), d, f))
-    env = dict(os.environ, VMOE_ROW_PAIR="1")
-    r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
-                       timeout=600)
-    assert r.returncode == 0 and "ROW_PAIR_OK" in r.stdout, r.stdout[-2000:] + r.stderr[-2000:]

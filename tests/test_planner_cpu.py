@@ -53,3 +53,38 @@ def test_refusals(vm):
         vm.vmoe_plan_slices([-1], [1.0], 4)
     assert e.value.status == vm.VMOE_ERR_INVALID
     assert vm.vmoe_plan_slices([], [], 4) == []
+
+
+@pytest.mark.parametrize("seed", range(40))
+def test_plan_shares_matches_oracle(vm, seed):
+    """vmoe_plan_shares (host C++) against the oracle's fill-clamp-refill rounded to
+    whole units (Section 3.2.2): identical shares on random instances, and on the
+    instances the budgeted backward builds (one expert per (task, expert) group of a
+    slice, work from its load, one to twelve SM pairs, 76 pairs)."""
+    rng = random.Random(500 + seed)
+    if seed % 2:
+        n = rng.randint(0, 30)
+        work = [rng.choice([0.0, rng.random() * 100, float(rng.randint(1, 9))]) for _ in range(n)]
+        mn = [rng.randint(0, 3) for _ in range(n)]
+        sat = [m + rng.randint(0, 10) for m in mn]
+        budget = sum(mn) + rng.randint(0, 60)
+    else:
+        n = rng.randint(1, 76)
+        loads = [rng.randint(0, 124) for _ in range(n)]
+        work = [12 * (3 * 256 * 256 * 2 + L * (768 * 2 + 1024)) for L in loads]
+        mn, sat, budget = [1] * n, [12] * n, 76
+    got = vm.vmoe_plan_shares(work, mn, sat, budget)
+    assert got == oracle.integer_shares(work, mn, sat, budget)
+
+
+def test_plan_shares_errors(vm):
+    with pytest.raises(vm.VmoeError) as ei:
+        vm.vmoe_plan_shares([1.0, 1.0], [3, 3], [5, 5], 5)  # minima above the budget
+    assert ei.value.status == vm.VMOE_ERR_UNSUPPORTED
+    with pytest.raises(vm.VmoeError) as ei:
+        vm.vmoe_plan_shares([1.0, float("nan")], [0, 0], [5, 5], 5)
+    assert ei.value.status == vm.VMOE_ERR_INVALID
+    with pytest.raises(vm.VmoeError) as ei:
+        vm.vmoe_plan_shares([1.0], [3], [2], 5)  # saturation below minimum
+    assert ei.value.status == vm.VMOE_ERR_INVALID
+    assert vm.vmoe_plan_shares([], [], [], 7) == []
