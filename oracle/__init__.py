@@ -22,6 +22,10 @@ Parity status (what pins each function, see ``tests/test_oracle_pins.py``):
                   gates differentiable) and central finite differences
   plan_slices     (planner.py, plain Python) brute-force subset enumeration, a
                   textbook knapsack instance, equal-weight closed forms
+  attention_expert_fwd / _bwd  (attention.py, numpy) torch float64 autograd
+                  through scaled_dot_product_attention, central finite
+                  differences, one-token and zero-query closed forms,
+                  permutation equivariance, padding rows and empty groups
   fill_clamp_refill / integer_shares  (planner.py) the closed form
                   min(sat, min + lambda w) with lambda found by bisection, a
                   hand-worked example (tests/golden/shares_example.json), sums
