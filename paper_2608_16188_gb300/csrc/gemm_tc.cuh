@@ -44,12 +44,31 @@ constexpr int BM = 128;  // rows of one MMA tile (TMEM lanes)
 constexpr int BK = 64;   // K per pipeline slot = one 128-byte swizzle row of bf16
 constexpr int THREADS = 320;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
 constexpr int EPI_WARP_BYTES = 32 * 80;  // 32 rows x (64 data + 16 pad) bytes
+
+// Row-mode epilogue of the one-SM grouped GEMM: the two-output epilogues
+// (FC1 + GELU, dA + GELU') run 16 epilogue warps (4 per TMEM lane quarter),
+// the plain store 8, all in 32-column chunks.  The two-output epilogues are
+// issue-bound at 8 warps (about 31 instructions per output element); 16 warps
+// leave room for 3 pipeline stages instead of 4, which the plain-store GEMMs,
+// bound by their operand stream, cannot spare.  Measured on GB300 (ms; 8 -> 16
+// warps): dA 0.536 -> 0.518 and FC1 0.485 -> 0.477 at the 17-task ViT-B step,
+// 0.370 -> 0.321 and 0.301 -> 0.285 at the 6-task one; FC2 / dX 0.425 ->
+// 0.433 / 0.434 -> 0.445 at 17 tasks, hence 8 there.  16-column chunks (4
+// stages with 16 warps) gained nothing.
 constexpr int EPI_WARP_BYTES_TMA = 2 * 4096;  // two 32 x 64 bf16 tiles, 128-byte swizzle
 constexpr int MAX_G = 1024;
 constexpr unsigned long long TIMEOUT_NS = 4000000000ull;
 
 enum { MODE_ROW = 0, MODE_WGRAD = 1 };
 enum { EPI_STORE = 0, EPI_GELU = 1, EPI_DGELU = 2 };
+
+constexpr int ROW_CH = 32;
+template <int MODE, int EPI>
+struct Roles {
+    static constexpr int EW = (MODE == 0 && EPI != EPI_STORE) ? 16 : 8;  // epilogue warps
+    static constexpr int NT = 64 + 32 * EW;  // threads: producer, MMA, epilogue
+    static constexpr int PITCH = 80;         // staging row pitch (bytes): 64 data + 16 pad
+};
 
 // Epilogue store path per mode.  TMA bulk tensor stores from 128-byte-
 // swizzled staging need 64 KB of shared memory, which leaves room for 3
@@ -68,15 +87,21 @@ struct Shape {
     // Weight-gradient tiles have K = load <= 2 slots, so 3 slots suffice and
     // leave room for the double-buffered 128-byte-swizzled TMA-store staging.
     static constexpr bool TMA_EPI = UseTmaStore<MODE, EPI>::value;
-    static constexpr int STAGES = TMA_EPI ? (BN == 256 ? 3 : 4) : (BN == 256 ? 4 : 6);
-    static constexpr int EPI_BYTES = TMA_EPI ? 8 * EPI_WARP_BYTES_TMA : 8 * EPI_WARP_BYTES;
+    static constexpr int NT = Roles<MODE, EPI>::NT;
+    static constexpr int EPI_BYTES =
+        TMA_EPI ? 8 * EPI_WARP_BYTES_TMA : Roles<MODE, EPI>::EW * 32 * Roles<MODE, EPI>::PITCH;
     static constexpr uint32_t A_BYTES = BM * BK * 2;
     static constexpr uint32_t B_BYTES = BN * BK * 2;
     static constexpr uint32_t STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr size_t FIXED = 1024 + EPI_BYTES + 16 + NT * 4 + (MAX_G + 1) * 4 + 8 * 21;
+    static constexpr int STAGES_FIT = (int)((232448 - FIXED) / STAGE_BYTES);
+    static constexpr int STAGES_MAX = TMA_EPI ? (BN == 256 ? 3 : 4) : (BN == 256 ? 4 : 6);
+    static constexpr int STAGES = STAGES_FIT < STAGES_MAX ? STAGES_FIT : STAGES_MAX;
     static constexpr uint32_t TMEM_COLS = 2 * BN;
     static constexpr int NUM_BARS = 2 * STAGES + 5;
     static constexpr size_t SMEM_BYTES = 1024 + (size_t)STAGES * STAGE_BYTES + EPI_BYTES +
-                                         NUM_BARS * 8 + 16 + THREADS * 4 + (MAX_G + 1) * 4;
+                                         NUM_BARS * 8 + 16 + NT * 4 + (MAX_G + 1) * 4;
+    static_assert(SMEM_BYTES <= 232448, "over the 227 KB shared-memory limit");
 };
 
 struct Args {
@@ -263,6 +288,15 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
           "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
         : "r"(taddr));
 }
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+        "%12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+          "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
 __device__ __forceinline__ void tmem_ld_wait() {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
@@ -346,12 +380,13 @@ __device__ __forceinline__ Tile decode_tile(const Args &a, const int *prefix, in
 }
 
 template <int BN, int MODE, bool A_MN, bool B_MN, int EPI>
-__global__ void __launch_bounds__(THREADS, 1)
+__global__ void __launch_bounds__(Roles<MODE, EPI>::NT, 1)
 grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                     const __grid_constant__ CUtensorMap tmD, const __grid_constant__ CUtensorMap tmD2,
                     const __grid_constant__ TailMaps tmAt, Args args) {
     using S = Shape<BN, MODE, EPI>;
     constexpr int STAGES = S::STAGES;
+    constexpr int NT = S::NT;
     constexpr uint32_t IDESC = idesc_bf16(BM, BN, A_MN, B_MN);
 
     extern __shared__ uint8_t smem_raw[];
@@ -362,7 +397,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     uint64_t *bars = reinterpret_cast<uint64_t *>(epi_base + S::EPI_BYTES);
     int *misc = reinterpret_cast<int *>(bars + S::NUM_BARS);  // [0] tmem base, [1] abort, [2] total
     int *scan_tmp = misc + 4;
-    int *prefix = scan_tmp + THREADS;
+    int *prefix = scan_tmp + NT;
 
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
     auto bar_full = [&](int s) { return smem_u32(bars + s); };
@@ -379,7 +414,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         }
         for (int a = 0; a < 2; ++a) {
             mbar_init(bar_tfull(a), 1);
-            mbar_init(bar_tempty(a), 8);
+            mbar_init(bar_tempty(a), Roles<MODE, EPI>::EW);
         }
         mbar_init(bar_drain, 1);
         misc[1] = 0;
@@ -400,7 +435,7 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
     int total;
     if (MODE == MODE_ROW) {
         const int G = args.G;
-        const int per = (G + THREADS - 1) / THREADS;
+        const int per = (G + NT - 1) / NT;
         const int g0 = min(G, tid * per), g1 = min(G, g0 + per);
         int local = 0;
         for (int g = g0; g < g1; ++g) {
@@ -410,8 +445,8 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         }
         scan_tmp[tid] = local;
         __syncthreads();
-        if (warp == 0) {  // exclusive scan of THREADS partials, THREADS/32 per lane
-            constexpr int PER = THREADS / 32;
+        if (warp == 0) {  // exclusive scan of NT partials, NT/32 per lane
+            constexpr int PER = NT / 32;
             int v[PER], s = 0;
 #pragma unroll
             for (int i = 0; i < PER; ++i) {
@@ -672,32 +707,40 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         __syncwarp();
     } else {
         // ------------------------------------------------------------ epilogue (row mode, st.global)
-        // Warps 2..9.  Warps w and w+4 share TMEM lane quarter q = w & 3 (rows
-        // 32q..32q+31 of the tile) and split its BN columns in halves; each
-        // thread owns one row and works through its half in 32-column chunks.
+        // Warps 2 .. EW+1.  Warp w works on TMEM lane quarter q = w & 3 (rows
+        // 32q .. 32q+31 of the tile), each thread owning one row; the EW / 4
+        // warps of a quarter take the tile's CH-column chunks in turn (warp j:
+        // chunks j, j + EW/4, ...).  Per chunk: tcgen05.ld, the fused
+        // elementwise step, bf16 packing into a per-warp staging tile, and
+        // coalesced, row-masked 16-byte stores.
+        constexpr int EW = Roles<MODE, EPI>::EW;
+        constexpr int WPQ = EW / 4;                 // warps per lane quarter
+        constexpr int CH = ROW_CH;                  // columns per chunk
+        constexpr int NCH = BN / CH;                // chunks per tile row
+        constexpr int PITCH = Roles<MODE, EPI>::PITCH;   // staging row pitch (bytes)
+        constexpr int PIECES = CH * 2 / 16;         // 16-byte pieces of a staged row
+        constexpr int RPI = 32 / PIECES;            // rows per store instruction
         const int ew = warp - 2;
         const int q = warp & 3;
-        const int half = ew >> 2;
-        constexpr int COLS = BN / 2;
-        constexpr int NCH = COLS / 32;
-        uint8_t *stg = epi_base + ew * EPI_WARP_BYTES;
+        const int jw = ew >> 2;
+        uint8_t *stg = epi_base + ew * 32 * PITCH;
         const bool tanh_form = args.gelu_tanh != 0;
-        const int sub_r = lane >> 2, sub_c = lane & 3;  // row-store mapping: 8 rows x 4 x 16 B
+        const int sub_r = lane / PIECES, sub_c = lane % PIECES;  // row-store mapping
         // EPI_DGELU: the H values of this thread's row for the current chunk,
         // loaded one chunk ahead (and across tiles) so the epilogue never waits
         // on a fresh global load.
-        uint4 hcur[4], hnxt[4];
-        auto load_h = [&](const Tile &tl, int c, uint4 (&dst)[4]) {
+        uint4 hcur[CH / 8], hnxt[CH / 8];
+        auto load_h = [&](const Tile &tl, int c, uint4 (&dst)[CH / 8]) {
             const int r0 = tl.m_blk * BM + q * 32;
             if (r0 + lane < tl.rows_valid) {
                 const uint4 *src = reinterpret_cast<const uint4 *>(
                     args.aux + (long long)tl.gr * args.sAux + (long long)(r0 + lane) * args.ldd +
-                    tl.n_blk * BN + half * COLS + c * 32);
+                    tl.n_blk * BN + c * CH);
 #pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = __ldg(src + i);
+                for (int i = 0; i < CH / 8; ++i) dst[i] = __ldg(src + i);
             } else {
 #pragma unroll
-                for (int i = 0; i < 4; ++i) dst[i] = make_uint4(0, 0, 0, 0);
+                for (int i = 0; i < CH / 8; ++i) dst[i] = make_uint4(0, 0, 0, 0);
             }
         };
         // Stage 32 packed rows of this warp and store them coalesced, masked to
@@ -705,17 +748,22 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
         auto store_rows = [&](__nv_bfloat16 *base, int nvalid) {
             __syncwarp();
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const int r = i * 8 + sub_r;
+            for (int i = 0; i < PIECES; ++i) {
+                const int r = i * RPI + sub_r;
                 if (r < nvalid)
                     *reinterpret_cast<uint4 *>(base + (long long)r * args.ldd + sub_c * 8) =
-                        *reinterpret_cast<const uint4 *>(stg + r * 80 + sub_c * 16);
+                        *reinterpret_cast<const uint4 *>(stg + r * PITCH + sub_c * 16);
             }
             __syncwarp();
         };
+        auto stage = [&](const float *v) {
+#pragma unroll
+            for (int i = 0; i < CH / 8; ++i)
+                *reinterpret_cast<uint4 *>(stg + lane * PITCH + i * 16) = f32_to_bf16x8(v + i * 8);
+        };
         int it = 0;
         Tile t = decode_tile<MODE>(args, prefix, blockIdx.x < total ? blockIdx.x : 0);
-        if (EPI == EPI_DGELU && blockIdx.x < total) load_h(t, 0, hcur);
+        if (EPI == EPI_DGELU && blockIdx.x < total) load_h(t, jw, hcur);
         for (int u = blockIdx.x; u < total; u += gridDim.x, ++it) {
             const bool have_next = u + (int)gridDim.x < total;
             const Tile tn = decode_tile<MODE>(args, prefix, have_next ? u + gridDim.x : u);
@@ -730,67 +778,57 @@ grouped_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_consta
             // residual) after its load rows; else the group's slab
             const bool cmpd = (args.compact & CMP_D) != 0;
             const long long gofs = (cmpd ? (long long)t.crow * args.ldd : (long long)t.gr * args.sD) +
-                                   (long long)row0 * args.ldd + t.n_blk * BN + half * COLS;
+                                   (long long)row0 * args.ldd + t.n_blk * BN;
             const long long gofs2 = cmpd ? gofs + (long long)t.rows_valid * args.ldd : gofs;
-            const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) +
-                                  (uint32_t)(acc * BN + half * COLS);
-            for (int c = 0; c < NCH; ++c) {
+            const uint32_t trow = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+#pragma unroll 1
+            for (int c = jw; c < NCH; c += WPQ) {
                 if (EPI == EPI_DGELU) {
-                    if (c + 1 < NCH) load_h(t, c + 1, hnxt);
-                    else if (have_next) load_h(tn, 0, hnxt);
+                    if (c + WPQ < NCH) load_h(t, c + WPQ, hnxt);
+                    else if (have_next) load_h(tn, jw, hnxt);
                 }
                 if (nvalid > 0) {
-                    float v[32];
+                    float v[CH];
                     if (t.kblocks > 0) {
-                        uint32_t r[32];
-                        tmem_ld32(trow + c * 32, r);
+                        uint32_t r[CH];
+                        if (CH == 32) tmem_ld32(trow + c * CH, *reinterpret_cast<uint32_t(*)[32]>(r));
+                        else tmem_ld16(trow + c * CH, *reinterpret_cast<uint32_t(*)[16]>(r));
                         tmem_ld_wait();
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+                        for (int i = 0; i < CH; ++i) v[i] = __uint_as_float(r[i]);
                     } else {
 #pragma unroll
-                        for (int i = 0; i < 32; ++i) v[i] = 0.0f;
+                        for (int i = 0; i < CH; ++i) v[i] = 0.0f;
                     }
                     if (EPI == EPI_DGELU) {
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
+                        for (int i = 0; i < CH / 8; ++i) {
                             float hv[8];
                             bf16x8_to_f32(hcur[i], hv);
 #pragma unroll
                             for (int e = 0; e < 8; ++e) v[i * 8 + e] *= gelu_deriv_fast(hv[e], tanh_form);
                         }
                     }
-#pragma unroll
-                    for (int i = 0; i < 4; ++i)
-                        *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(v + i * 8);
-                    store_rows(args.D + gofs + c * 32, nvalid);
+                    stage(v);
+                    store_rows(args.D + gofs + c * CH, nvalid);
                     if (EPI == EPI_DGELU) {  // residual v - bf16(v): dH = hi + lo to ~16 bits
+                        float lv[CH];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float lv[8];
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) {
-                                const float x = v[i * 8 + e];
-                                lv[e] = x - __bfloat162float(__float2bfloat16_rn(x));
-                            }
-                            *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(lv);
-                        }
-                        store_rows(args.D2 + gofs2 + c * 32, nvalid);
+                        for (int i = 0; i < CH; ++i) lv[i] = v[i] - __bfloat162float(__float2bfloat16_rn(v[i]));
+                        stage(lv);
+                        store_rows(args.D2 + gofs2 + c * CH, nvalid);
                     }
                     if (EPI == EPI_GELU) {
+                        float gv[CH];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            float gv[8];
-#pragma unroll
-                            for (int e = 0; e < 8; ++e) gv[e] = gelu_fast(v[i * 8 + e], tanh_form);
-                            *reinterpret_cast<uint4 *>(stg + lane * 80 + i * 16) = f32_to_bf16x8(gv);
-                        }
-                        store_rows(args.D2 + gofs2 + c * 32, nvalid);
+                        for (int i = 0; i < CH; ++i) gv[i] = gelu_fast(v[i], tanh_form);
+                        stage(gv);
+                        store_rows(args.D2 + gofs2 + c * CH, nvalid);
                     }
                 }
                 if (EPI == EPI_DGELU) {
 #pragma unroll
-                    for (int i = 0; i < 4; ++i) hcur[i] = hnxt[i];
+                    for (int i = 0; i < CH / 8; ++i) hcur[i] = hnxt[i];
                 }
             }
             tc_fence_before();
@@ -1186,7 +1224,7 @@ int launch(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &md,
     if (max_tiles <= 0) return VMOE_OK;
     long long grid = max_tiles < num_sms() ? max_tiles : num_sms();
     trace_before(s, name);
-    const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(THREADS), S::SMEM_BYTES, s, ma, mb,
+    const int st = launch_kernel(kern, dim3((unsigned)grid), dim3(S::NT), S::SMEM_BYTES, s, ma, mb,
                                  md, md2, mat, a);
     trace_after(s);
     return st;

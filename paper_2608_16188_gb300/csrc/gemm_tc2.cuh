@@ -1037,7 +1037,13 @@ int row_gemm(const Dims &p, const __nv_bfloat16 *act, int K, const __nv_bfloat16
              cudaStream_t s, const char *name, long long sD = 0, long long sAux = 0,
              long long sAct = 0, const Slice &sl = Slice()) {
     const int G = p.G(), C = p.C;
-    const bool wide = N % 256 == 0;
+    // 256-column tiles, or 128 when N needs it -- and, for a plain-store GEMM,
+    // when 256-column tiles would give the SMs fewer than two waves (the slices
+    // of the memory-budgeted backward: dX over ~70 groups is 204 wide tiles on
+    // 152 SMs); the tile width does not change any output element's sums
+    const int entries = sl.n > 0 ? sl.n : G;
+    const long long wide_tiles = (long long)entries * ((C + BM - 1) / BM) * (N / 256);
+    const bool wide = N % 256 == 0 && !(EPI == EPI_STORE && wide_tiles < 2LL * num_sms());
     const int BN = wide ? 256 : 128;
     const bool pair = row_pair_enabled() && C > BM;
     const int bcols = pair ? BN / 2 : BN;  // B columns one CTA loads
