@@ -173,7 +173,7 @@ __device__ __forceinline__ void rm_ldsm_x4(uint32_t (&r)[4], const void *smem) {
 
 // NB blocks of 8 experts per pass (NB even).
 template <int NB>
-__global__ void __launch_bounds__(RM_THREADS, NB >= 8 ? 2 : 3)
+__global__ void __launch_bounds__(RM_THREADS, 3)
 route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__restrict__ wr,
                  const float *__restrict__ bias, float *__restrict__ logits,
                  int32_t *__restrict__ out_idx, float *__restrict__ out_gate) {
@@ -252,15 +252,11 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
     const __nv_bfloat16 *xa = xs + (warp * 16 + (lane & 15)) * RM_XP + (lane >> 4) * 8;
     const __nv_bfloat16 *wb = ws + ((lane & 7) + (lane >> 4) * 8) * RM_XP + ((lane >> 3) & 1) * 8;
     for (int e0 = 0; e0 < E; e0 += NP) {
-        // one accumulator per weight part: three independent MMA chains per
-        // output fragment instead of one chain three MMAs deep per k step
-        float acc[3][NB][4];
+        float acc[NB][4];
 #pragma unroll
-        for (int sp = 0; sp < 3; ++sp)
+        for (int nb = 0; nb < NB; ++nb)
 #pragma unroll
-            for (int nb = 0; nb < NB; ++nb)
-#pragma unroll
-                for (int i = 0; i < 4; ++i) acc[sp][nb][i] = 0.0f;
+            for (int i = 0; i < 4; ++i) acc[nb][i] = 0.0f;
         load_chunk(e0, 0);
         for (int k0 = 0; k0 < d; k0 += RM_KC) {
             __syncthreads();  // the previous chunk's fragments have been read
@@ -277,11 +273,10 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
 #pragma unroll
                     for (int sp = 0; sp < 3; ++sp) rm_ldsm_x4(b[sp], wb + (sp * NP + np * 16) * RM_XP + ks);
 #pragma unroll
-                    for (int sp = 0; sp < 3; ++sp)
+                    for (int h = 0; h < 2; ++h)
 #pragma unroll
-                        for (int h = 0; h < 2; ++h)
-                            mma_bf16_16816(acc[sp][2 * np + h], a[0], a[1], a[2], a[3], b[sp][2 * h],
-                                           b[sp][2 * h + 1]);
+                        for (int sp = 2; sp >= 0; --sp)  // smallest part first
+                            mma_bf16_16816(acc[2 * np + h], a[0], a[1], a[2], a[3], b[sp][2 * h], b[sp][2 * h + 1]);
                 }
             }
         }
@@ -291,9 +286,7 @@ route_mma_kernel(Dims p, const __nv_bfloat16 *__restrict__ x, const float *__res
             for (int i = 0; i < 4; ++i) {
                 const int r = warp * 16 + g + (i >> 1) * 8;
                 const int e = e0 + nb * 8 + 2 * tq + (i & 1);
-                // the parts' sums, smallest first
-                const float v = (acc[2][nb][i] + acc[1][nb][i]) + acc[0][nb][i];
-                if (r < ntok && e < E) lg[r * ldl + e] = v + (bias ? bias[(long long)t * E + e] : 0.0f);
+                if (r < ntok && e < E) lg[r * ldl + e] = acc[nb][i] + (bias ? bias[(long long)t * E + e] : 0.0f);
             }
     }
     __syncthreads();
