@@ -437,6 +437,71 @@ def measure_secondary(vm, cfg, dev, stream, steps, warmup, peaks, seed):
     return out
 
 
+def measure_attention(vm, cfg, heads, dev, stream, steps, warmup, peaks, seed):
+    """The attention-expert variant of the step at cfg's shape: route, dispatch,
+    vmoe_attn_expert_fwd, combine, weighted dispatch of dY, vmoe_attn_expert_bwd,
+    combine of dX -- H-head attention (head dimension 64) among each group's
+    routed tokens in place of the FFN experts.  Weights drawn on the device."""
+    import torch
+    p = vm.problem(cfg.T, cfg.N, cfg.d, cfg.f, cfg.E, cfg.k, cfg.cf, cfg.dtype, cfg.flags)
+    C = vm.vmoe_problem_capacity(p)
+    inp = workloads.make_inputs(cfg.with_(capacity=C), with_weights=False)
+    inp = {k2: (None if v is None else v.to(dev)) for k2, v in inp.items()}
+    hd = heads * 64
+    g = torch.Generator(device=dev)
+    g.manual_seed(seed)
+    G, d = cfg.T * cfg.E, cfg.d
+    wqkv = (torch.randn((G, d, 3 * hd), generator=g, device=dev) / d ** 0.5).to(torch.bfloat16)
+    wo = (torch.randn((G, hd, d), generator=g, device=dev) / hd ** 0.5).to(torch.bfloat16)
+    b = vm.Buffers(p)
+    e = lambda *sh, dt=torch.bfloat16: torch.empty(sh, dtype=dt, device=dev)  # noqa: E731
+    qkv, o, ye, lse = e(G, C, 3 * hd), e(G, C, hd), e(G, C, d), e(G, heads, C, dt=torch.float32)
+    dxe, dwqkv, dwo = e(G, C, d), e(G, d, 3 * hd), e(G, hd, d)
+    ws = torch.empty(vm.vmoe_attn_expert_bwd_workspace_size(p, heads), dtype=torch.uint8, device=dev)
+
+    def step(st):
+        vm.vmoe_route(p, inp["x"], inp["w_router"], inp["bias"], b.logits, b.idx, b.gate, b.slot, b.load, st)
+        vm.vmoe_dispatch(p, inp["x"], None, b.idx, b.slot, b.load, b.xe, st)
+        vm.vmoe_attn_expert_fwd(p, heads, b.xe, wqkv, wo, b.load, qkv, o, lse, ye, st)
+        vm.vmoe_combine(p, ye, b.gate, b.idx, b.slot, b.y, st)
+        vm.vmoe_dispatch(p, inp["dy"], b.gate, b.idx, b.slot, b.load, b.dye, st)
+        vm.vmoe_attn_expert_bwd(p, heads, b.xe, qkv, o, lse, wqkv, wo, b.dye, b.load, dxe, dwqkv, dwo, ws,
+                                stream=st)
+        vm.vmoe_combine(p, dxe, None, b.idx, b.slot, b.dx, st)
+    for _ in range(warmup):
+        step(stream)
+    torch.cuda.synchronize(dev)
+    loads = b.load.flatten().tolist()
+    ms = time_steps(step, stream, steps) / steps
+    per_kernel, _ = traced_kernels(vm, step, stream, min(steps, 20))
+    st = vm.vmoe_device_status()
+    if st != 0:
+        raise RuntimeError("device status after the attention experts: " + vm.status_string(st))
+    A = int(sum(loads))
+    sq = float(sum(L * L for L in loads))
+    # flops on kept rows: projections 2 A d (3 hd + hd) forward, twice that backward;
+    # the core 4 sum(L^2) hd forward (S and P V), 8 sum(L^2) hd backward (recomputed
+    # S, dP, dQ, dK, dV minus the shared S)
+    proj = 2.0 * A * d * 4 * hd
+    core = 4.0 * sq * hd
+    kst = {}
+    for name, lst in per_kernel.items():
+        kst[name] = {"launches": len(lst), "ms_avg": round(sum(lst) / len(lst), 5)}
+    core_ms = sum(kst[n]["ms_avg"] for n in ("attn_fwd", "attn_bwd_dq", "attn_bwd_dkv") if n in kst)
+    out = {"config": {"workload": cfg.name + " shape with attention experts (H=%d, head dim 64)" % heads,
+                      "T": cfg.T, "tokens_per_task": cfg.N, "d_model": d, "E": cfg.E, "k": cfg.k,
+                      "capacity": C, "heads": heads, "kept_assignments": A},
+           "value": round(cfg.T * cfg.N / (ms * 1e-3), 1), "unit": UNIT, "ms_per_step": round(ms, 5),
+           "steps": steps,
+           "tflops": round((3 * proj + 3 * core) / (ms * 1e-3) / 1e12, 2),
+           "core_ms_per_step": round(core_ms, 5),
+           "core_tflop_s": round(3 * core / (core_ms * 1e-3) / 1e12, 2) if core_ms else None,
+           "kernels": kst}
+    del b, qkv, o, ye, dxe, dwqkv, dwo, ws, wqkv, wo
+    torch.cuda.empty_cache()
+    return out
+
+
 def run_ours(args, cfg, rank, world, local_rank):
     import torch
     import paper_2608_16188_gb300 as vm
@@ -666,6 +731,8 @@ def run_ours(args, cfg, rank, world, local_rank):
         out["workloads"] = {name: measure_secondary(vm, workloads.CONFIGS[name], dev, stream,
                                                     args.aux_steps, args.warmup, peaks, seed=7)
                             for name in SECONDARY if name != cfg.name}
+        out["attention_experts"] = measure_attention(vm, workloads.CONFIGS[workloads.HEADLINE], 12, dev,
+                                                     stream, args.aux_steps, args.warmup, peaks, seed=9)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(cfg, budget_s=args.cpu_budget)
     if dist is not None:

@@ -215,6 +215,47 @@ int vmoe_expert_bwd_static_scratch(const vmoe_problem *p, const void *xe, const 
                                    const int32_t *load, void *dxe, void *dw1, void *dw2,
                                    void *cuda_stream);
 
+/* Attention experts (Section 2.1: V-MoE expertizes the ViT's attention as well
+ * as its MLP; Section 3.2.1's memory estimator gives such an expert buffers of
+ * order T d_k for Q / K / V and T^2 for the scores).  The paper gives no more;
+ * the library's reading: each (task, expert) group g owns W_qkv [d, 3 H 64]
+ * (column blocks Q | K | V, head h at columns h * 64 of each) and W_o [H 64, d],
+ * and runs H-head softmax attention, head dimension 64, among its L = load[g]
+ * routed tokens only (the rows [0, L) of xe, as dispatched by vmoe_dispatch):
+ *   QKV = Xe W_qkv;  per head  S = Q_h K_h^T / 8,  P = softmax over the L keys
+ *   (row maximum subtracted),  O_h = P V_h;  Ye = O W_o,
+ * then vmoe_combine gate-weights Ye back to token order as for the FFN.
+ * bf16 only, H even, d % 128 == 0, C <= 512 (else VMOE_ERR_UNSUPPORTED);
+ * p->d_ff is not used.  Sums accumulate in fp32; P is rounded to bf16 for the
+ * P V product; no atomics.  Rows s >= load[g] of xe (and of dye, qkv, o in the
+ * backward) are padding, reach no output and are not written.
+ *   xe [T,E,C,d], wqkv [T,E,d,3H64], wo [T,E,H64,d] in; qkv [T,E,C,3H64],
+ *   o [T,E,C,H64] bf16 and lse [T,E,H,C] fp32 (each row's log-sum-exp of the
+ *   scaled scores, kept for the backward) out; ye [T,E,C,d] out. */
+int vmoe_attn_expert_fwd(const vmoe_problem *p, int heads, const void *xe, const void *wqkv,
+                         const void *wo, const int32_t *load, void *qkv, void *o, float *lse, void *ye,
+                         void *cuda_stream);
+
+/* Workspace of vmoe_attn_expert_bwd in bytes (dO and dQKV in bf16, then the row
+ * sums D of dO * O in fp32), or 0 for an invalid or unsupported problem. */
+size_t vmoe_attn_expert_bwd_workspace_size(const vmoe_problem *p, int heads);
+
+/* Backward of vmoe_attn_expert_fwd with routing and gates fixed: the gradient
+ * of <dYe, Ye> per group,
+ *   dO = dYe W_o^T,  dW_o = O^T dYe,  D = rowsum(dO * O) per head,
+ *   dS = P * (dO_h V_h^T - D),  dQ_h = dS K_h / 8,  dK_h = dS^T Q_h / 8,  dV_h = P^T dO_h,
+ *   dXe = dQKV W_qkv^T,  dW_qkv = Xe^T dQKV,
+ * P rebuilt from qkv and lse.  Inputs as written by the forward (xe, qkv, o, lse)
+ * and dye [T,E,C,d] (vmoe_dispatch of dY with the gates); outputs dxe [T,E,C,d]
+ * (rows >= load not written), dwqkv [T,E,d,3H64] and dwo [T,E,H64,d] (zero for an
+ * empty group).  workspace: caller-owned device scratch of at least
+ * vmoe_attn_expert_bwd_workspace_size(p, heads) bytes (else VMOE_ERR_INVALID),
+ * its contents clobbered.  Asynchronous on `cuda_stream`. */
+int vmoe_attn_expert_bwd(const vmoe_problem *p, int heads, const void *xe, const void *qkv,
+                         const void *o, const float *lse, const void *wqkv, const void *wo,
+                         const void *dye, const int32_t *load, void *dxe, void *dwqkv, void *dwo,
+                         void *workspace, size_t workspace_bytes, void *cuda_stream);
+
 /* Combine back to token order: dst[t,n,:] = sum over kept choices j (slot >= 0)
  * of w * src[t, expert_idx_j, slot_j, :], w = weight[t,n,j] or 1 if NULL,
  * summed in fp32 in the order j = 0..k-1 and rounded once; a token with every

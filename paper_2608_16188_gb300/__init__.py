@@ -36,6 +36,7 @@ EXPORTS = ("vmoe_version", "vmoe_status_string", "vmoe_problem_capacity", "vmoe_
            "vmoe_dispatch", "vmoe_expert_fwd", "vmoe_expert_bwd_workspace_size",
            "vmoe_expert_bwd_min_workspace_size",
            "vmoe_expert_bwd", "vmoe_expert_bwd_static_scratch", "vmoe_combine", "vmoe_router_bwd", "vmoe_plan_slices", "vmoe_plan_shares",
+           "vmoe_attn_expert_fwd", "vmoe_attn_expert_bwd", "vmoe_attn_expert_bwd_workspace_size",
            "vmoe_device_status", "vmoe_selftest_bounded_wait", "vmoe_trace_enable",
            "vmoe_trace_disable", "vmoe_trace_get")
 
@@ -81,6 +82,9 @@ def library():
             "vmoe_expert_bwd_static_scratch": (ctypes.c_int, [PP] + [_P] * 10 + [_P]),
             "vmoe_combine": (ctypes.c_int, [PP] + [_P] * 5 + [_P]),
             "vmoe_router_bwd": (ctypes.c_int, [PP] + [_P] * 13 + [_P]),
+            "vmoe_attn_expert_fwd": (ctypes.c_int, [PP, ctypes.c_int] + [_P] * 9),
+            "vmoe_attn_expert_bwd_workspace_size": (ctypes.c_size_t, [PP, ctypes.c_int]),
+            "vmoe_attn_expert_bwd": (ctypes.c_int, [PP, ctypes.c_int] + [_P] * 12 + [ctypes.c_size_t, _P]),
             "vmoe_plan_slices": (ctypes.c_int, [ctypes.c_int, _P, _P, ctypes.c_int64,
                                                 ctypes.c_double, ctypes.c_double, _P, _P]),
             "vmoe_plan_shares": (ctypes.c_int, [ctypes.c_int, _P, _P, _P, ctypes.c_int32, _P]),
@@ -197,6 +201,28 @@ def vmoe_expert_bwd_static_scratch(p, xe, h, a, w1, w2, dye, load, dxe, dw1, dw2
 def vmoe_combine(p, src, weight, expert_idx, slot, dst, stream=None):
     _check(library().vmoe_combine(ctypes.byref(p), _ptr(src), _ptr(weight), _ptr(expert_idx),
                                   _ptr(slot), _ptr(dst), _stream(stream)), "vmoe_combine")
+
+
+def vmoe_attn_expert_fwd(p, heads, xe, wqkv, wo, load, qkv, o, lse, ye, stream=None):
+    """Attention experts, forward (see include/vmoe.h)."""
+    _check(library().vmoe_attn_expert_fwd(ctypes.byref(p), int(heads), _ptr(xe), _ptr(wqkv), _ptr(wo),
+                                          _ptr(load), _ptr(qkv), _ptr(o), _ptr(lse), _ptr(ye),
+                                          _stream(stream)), "vmoe_attn_expert_fwd")
+
+
+def vmoe_attn_expert_bwd_workspace_size(p, heads) -> int:
+    return int(library().vmoe_attn_expert_bwd_workspace_size(ctypes.byref(p), int(heads)))
+
+
+def vmoe_attn_expert_bwd(p, heads, xe, qkv, o, lse, wqkv, wo, dye, load, dxe, dwqkv, dwo, workspace,
+                         workspace_bytes=None, stream=None):
+    """Attention experts, backward (see include/vmoe.h)."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(library().vmoe_attn_expert_bwd(
+        ctypes.byref(p), int(heads), _ptr(xe), _ptr(qkv), _ptr(o), _ptr(lse), _ptr(wqkv), _ptr(wo),
+        _ptr(dye), _ptr(load), _ptr(dxe), _ptr(dwqkv), _ptr(dwo), _ptr(workspace), int(workspace_bytes),
+        _stream(stream)), "vmoe_attn_expert_bwd")
 
 
 def vmoe_router_bwd(p, x, w_router, logits, expert_idx, gate, slot, dy, ye, dgate, dlogits,

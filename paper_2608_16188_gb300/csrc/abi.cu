@@ -298,6 +298,57 @@ int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const 
                                  (float *)dxe, (float *)dw1, (float *)dw2, (float *)workspace, s);
 }
 
+// Attention experts: bf16, head dimension 64, an even number of heads (the
+// projection GEMMs need H * 64 to be a multiple of 128), d % 128 == 0, C <= 512.
+static int check_attn(const vmoe_problem *p, int heads, Dims *d) {
+    int st = check_problem(p, d);
+    if (st != VMOE_OK) return st;
+    if (heads < 1) return VMOE_ERR_INVALID;
+    if (!d->bf16 || heads % 2 != 0 || d->d % 128 != 0 || !attn_core_supported(d->C, 64))
+        return VMOE_ERR_UNSUPPORTED;
+    if ((long long)d->C * 3 * heads * 64 >= (1LL << 31)) return VMOE_ERR_UNSUPPORTED;
+    return VMOE_OK;
+}
+
+int vmoe_attn_expert_fwd(const vmoe_problem *p, int heads, const void *xe, const void *wqkv,
+                         const void *wo, const int32_t *load, void *qkv, void *o, float *lse, void *ye,
+                         void *cuda_stream) {
+    Dims d;
+    int st = check_attn(p, heads, &d);
+    if (st != VMOE_OK) return st;
+    if (!dev_ok(xe) || !dev_ok(wqkv) || !dev_ok(wo) || !dev_ok(load) || !dev_ok(qkv) || !dev_ok(o) ||
+        !dev_ok(lse) || !dev_ok(ye))
+        return VMOE_ERR_INVALID;
+    return launch_attn_expert_fwd(d, heads, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)wqkv,
+                                  (const __nv_bfloat16 *)wo, load, (__nv_bfloat16 *)qkv, (__nv_bfloat16 *)o,
+                                  lse, (__nv_bfloat16 *)ye, (cudaStream_t)cuda_stream);
+}
+
+size_t vmoe_attn_expert_bwd_workspace_size(const vmoe_problem *p, int heads) {
+    Dims d;
+    if (check_attn(p, heads, &d) != VMOE_OK) return 0;
+    return attn_bwd_workspace(d, heads);
+}
+
+int vmoe_attn_expert_bwd(const vmoe_problem *p, int heads, const void *xe, const void *qkv,
+                         const void *o, const float *lse, const void *wqkv, const void *wo,
+                         const void *dye, const int32_t *load, void *dxe, void *dwqkv, void *dwo,
+                         void *workspace, size_t workspace_bytes, void *cuda_stream) {
+    Dims d;
+    int st = check_attn(p, heads, &d);
+    if (st != VMOE_OK) return st;
+    if (!dev_ok(xe) || !dev_ok(qkv) || !dev_ok(o) || !dev_ok(lse) || !dev_ok(wqkv) || !dev_ok(wo) ||
+        !dev_ok(dye) || !dev_ok(load) || !dev_ok(dxe) || !dev_ok(dwqkv) || !dev_ok(dwo) ||
+        !dev_ok(workspace))
+        return VMOE_ERR_INVALID;
+    if (workspace_bytes < attn_bwd_workspace(d, heads)) return VMOE_ERR_INVALID;
+    return launch_attn_expert_bwd(d, heads, (const __nv_bfloat16 *)xe, (const __nv_bfloat16 *)qkv,
+                                  (const __nv_bfloat16 *)o, lse, (const __nv_bfloat16 *)wqkv,
+                                  (const __nv_bfloat16 *)wo, (const __nv_bfloat16 *)dye, load,
+                                  (__nv_bfloat16 *)dxe, (__nv_bfloat16 *)dwqkv, (__nv_bfloat16 *)dwo,
+                                  workspace, (cudaStream_t)cuda_stream);
+}
+
 int vmoe_device_status(int reset) {
     if (cudaDeviceSynchronize() != cudaSuccess) return VMOE_ERR_CUDA;
     int *addr = device_status_word();

@@ -107,6 +107,24 @@ int launch_router_bwd(const Dims &p, const void *x, const float *w_router, const
                       const void *ye, float *dgate, float *dlogits, float *dw_router, float *dbias,
                       void *dx, cudaStream_t s);
 
+// Attention experts (attention.cu: the attention core; gemm_tc_fwd.cu /
+// gemm_tc_bwd.cu: the projections and their gradients).  Head dimension 64.
+bool attn_core_supported(int C, int head_dim);
+int launch_attn_core_fwd(int G, int C, int H, const int32_t *load, const __nv_bfloat16 *qkv,
+                         __nv_bfloat16 *o, float *lse, cudaStream_t s);
+int launch_attn_core_bwd(int G, int C, int H, const int32_t *load, const __nv_bfloat16 *qkv,
+                         const __nv_bfloat16 *o, const float *lse, const __nv_bfloat16 *dout, float *dsum,
+                         __nv_bfloat16 *dqkv, cudaStream_t s);
+int launch_attn_expert_fwd(const Dims &p, int H, const __nv_bfloat16 *xe, const __nv_bfloat16 *wqkv,
+                           const __nv_bfloat16 *wo, const int32_t *load, __nv_bfloat16 *qkv,
+                           __nv_bfloat16 *o, float *lse, __nv_bfloat16 *ye, cudaStream_t s);
+size_t attn_bwd_workspace(const Dims &p, int H);
+int launch_attn_expert_bwd(const Dims &p, int H, const __nv_bfloat16 *xe, const __nv_bfloat16 *qkv,
+                           const __nv_bfloat16 *o, const float *lse, const __nv_bfloat16 *wqkv,
+                           const __nv_bfloat16 *wo, const __nv_bfloat16 *dye, const int32_t *load,
+                           __nv_bfloat16 *dxe, __nv_bfloat16 *dwqkv, __nv_bfloat16 *dwo, void *workspace,
+                           cudaStream_t s);
+
 // ---------------------------------------------------------------------------
 // Device helpers.
 

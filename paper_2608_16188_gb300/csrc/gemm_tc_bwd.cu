@@ -197,4 +197,34 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
     return st;
 }
 
+// Attention experts, backward: dO = dYe W_o^T, dW_o = O^T dYe, the attention
+// core's dQ, dK, dV (attention.cu) into dQKV, dXe = dQKV W_qkv^T and
+// dW_qkv = Xe^T dQKV.  The workspace holds dO [G, C, H dk] and dQKV
+// [G, C, 3 H dk] (bf16), then D [G, H, C] (fp32).
+size_t attn_bwd_workspace(const Dims &p, int H) {
+    const size_t hd = (size_t)H * 64, rows = (size_t)p.G() * p.C;
+    return rows * hd * 2 + rows * 3 * hd * 2 + (size_t)p.G() * H * p.C * 4;
+}
+
+int launch_attn_expert_bwd(const Dims &p, int H, const __nv_bfloat16 *xe, const __nv_bfloat16 *qkv,
+                           const __nv_bfloat16 *o, const float *lse, const __nv_bfloat16 *wqkv,
+                           const __nv_bfloat16 *wo, const __nv_bfloat16 *dye, const int32_t *load,
+                           __nv_bfloat16 *dxe, __nv_bfloat16 *dwqkv, __nv_bfloat16 *dwo, void *workspace,
+                           cudaStream_t s) {
+    const int hd = H * 64;
+    const size_t rows = (size_t)p.G() * p.C;
+    __nv_bfloat16 *dout = static_cast<__nv_bfloat16 *>(workspace);
+    __nv_bfloat16 *dqkv = dout + rows * hd;
+    float *dsum = reinterpret_cast<float *>(dqkv + rows * 3 * hd);
+    int st = row_gemm<EPI_STORE, false>(p, dye, p.d, wo, hd, load, dout, nullptr, nullptr, s, "attn_dout");
+    if (st != VMOE_OK) return st;
+    if ((st = wgrad_gemm(p, o, hd, dye, p.d, load, dwo, s, "attn_dwo")) != VMOE_OK) return st;
+    if ((st = launch_attn_core_bwd(p.G(), p.C, H, load, qkv, o, lse, dout, dsum, dqkv, s)) != VMOE_OK)
+        return st;
+    if ((st = row_gemm<EPI_STORE, false>(p, dqkv, 3 * hd, wqkv, p.d, load, dxe, nullptr, nullptr, s,
+                                         "attn_dxe")) != VMOE_OK)
+        return st;
+    return wgrad_gemm(p, xe, p.d, dqkv, 3 * hd, load, dwqkv, s, "attn_dwqkv");
+}
+
 }  // namespace vmoe

@@ -67,4 +67,16 @@ int launch_expert_fwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bf
     return row_gemm<EPI_STORE, true>(p, act, p.f, w2, p.d, load, ye, nullptr, nullptr, s, "tc_fc2");
 }
 
+// Attention experts, forward: QKV = Xe W_qkv, the attention core (O and the
+// row log-sum-exp, attention.cu), Ye = O W_o.
+int launch_attn_expert_fwd(const Dims &p, int H, const __nv_bfloat16 *xe, const __nv_bfloat16 *wqkv,
+                           const __nv_bfloat16 *wo, const int32_t *load, __nv_bfloat16 *qkv,
+                           __nv_bfloat16 *o, float *lse, __nv_bfloat16 *ye, cudaStream_t s) {
+    const int hd = H * 64;
+    int st = row_gemm<EPI_STORE, true>(p, xe, p.d, wqkv, 3 * hd, load, qkv, nullptr, nullptr, s, "attn_qkv");
+    if (st != VMOE_OK) return st;
+    if ((st = launch_attn_core_fwd(p.G(), p.C, H, load, qkv, o, lse, s)) != VMOE_OK) return st;
+    return row_gemm<EPI_STORE, true>(p, o, hd, wo, p.d, load, ye, nullptr, nullptr, s, "attn_out");
+}
+
 }  // namespace vmoe

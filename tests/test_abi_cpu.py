@@ -123,3 +123,23 @@ def test_null_and_misaligned_pointers_are_rejected_without_cuda(vm):
     assert vm.vmoe_expert_bwd_workspace_size(p) == 2 * 4 * oracle.capacity(64, 4, 2, 1.25) * 256 * 2 * 2
     for s in (0, -1, -2, -3, -4, 7):
         assert isinstance(vm.status_string(s), str) and vm.status_string(s)
+
+
+def test_attention_expert_arguments_rejected_on_host(vm):
+    """Attention experts: bf16, an even head count, d % 128 == 0 and C <= 512, else
+    VMOE_ERR_UNSUPPORTED; null pointers and a short workspace are VMOE_ERR_INVALID."""
+    lib = vm.library()
+    P = 1 << 20
+    p = vm.problem(2, 300, 256, 1, 4, 2, 1.25, "bf16")
+    ws = vm.vmoe_attn_expert_bwd_workspace_size(p, 2)
+    C = oracle.capacity(300, 4, 2, 1.25)
+    assert ws == 8 * C * 128 * 2 + 8 * C * 384 * 2 + 8 * 2 * C * 4  # dO, dQKV, D
+    assert lib.vmoe_attn_expert_fwd(ctypes.byref(p), 2, P, P, P, P, P, P, P, None, None) == vm.VMOE_ERR_INVALID
+    assert lib.vmoe_attn_expert_fwd(ctypes.byref(p), 3, P, P, P, P, P, P, P, P, None) == vm.VMOE_ERR_UNSUPPORTED
+    assert lib.vmoe_attn_expert_fwd(ctypes.byref(p), 0, P, P, P, P, P, P, P, P, None) == vm.VMOE_ERR_INVALID
+    pf = vm.problem(2, 300, 256, 1, 4, 2, 1.25, "f32")
+    assert lib.vmoe_attn_expert_fwd(ctypes.byref(pf), 2, P, P, P, P, P, P, P, P, None) == vm.VMOE_ERR_UNSUPPORTED
+    wide = vm.problem(1, 4096, 256, 1, 2, 1, 1.0, "bf16")  # C = 2048 > 512
+    assert vm.vmoe_attn_expert_bwd_workspace_size(wide, 2) == 0
+    args = [P] * 12
+    assert lib.vmoe_attn_expert_bwd(ctypes.byref(p), 2, *args, ws - 1, None) == vm.VMOE_ERR_INVALID
