@@ -141,7 +141,7 @@ def traffic_record(kernel, workload, algo_bytes, path=None):
 
 # Source files behind each kernel name of the trace (for the traffic record's hash).
 KERNEL_SOURCES = {
-    "route_topk": ["route.cu", "topk.cuh", "common.cuh"],
+    "route_topk": ["route.cu", "route_tc.cu", "topk.cuh", "gemm_tc.cuh", "common.cuh"],
     "capacity_scan": ["route.cu", "common.cuh"],
     "dispatch": ["permute.cu", "common.cuh"],
     "combine": ["permute.cu", "common.cuh"],

@@ -53,6 +53,14 @@ bool shares_enabled() {
     return on;
 }
 
+bool route_tc_enabled() {
+    static const bool on = [] {
+        const char *v = getenv("VMOE_ROUTE_TC");
+        return v && v[0] == '1';
+    }();
+    return on;
+}
+
 bool row_pair_enabled() {
     static const bool on = [] {
         const char *v = getenv("VMOE_ROW_PAIR");

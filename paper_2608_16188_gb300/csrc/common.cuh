@@ -52,6 +52,9 @@ bool row_pair_enabled();
 // The fill-clamp-refill pair shares of the memory-budgeted backward's dW1,
 // off unless VMOE_SHARES=1 (abi.cu).
 bool shares_enabled();
+// The tcgen05 router for bf16 tokens (route_tc.cu), off unless
+// VMOE_ROUTE_TC=1; problems it does not take use the mma.sync router.
+bool route_tc_enabled();
 
 template <typename... KArgs, typename... Args>
 int launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t s,
@@ -71,6 +74,9 @@ int launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cu
 }
 
 // Launchers (one file each).
+int route_tc_width(const Dims &p);  // 0: the tcgen05 router does not take p
+int launch_route_tc(const Dims &p, const __nv_bfloat16 *x, const float *wr, const float *bias, float *logits,
+                    int32_t *idx, float *gate, cudaStream_t s);
 int launch_route(const Dims &p, const void *x, const float *w_router, const float *bias,
                  float *logits, int32_t *idx, float *gate, int32_t *slot, int32_t *load,
                  cudaStream_t s);

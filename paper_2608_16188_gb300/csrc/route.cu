@@ -2,7 +2,8 @@
 // capacity scan (Section 2.1 routing, Challenge #1 capacity limits,
 // Section 3.3.1 sequential assignment).
 //
-// Kernel 1 (route_topk), bf16 tokens: route_mma_kernel below -- the router
+// Kernel 1 (route_topk), bf16 tokens: route_mma_kernel below (or, with
+// VMOE_ROUTE_TC=1, route_tc_kernel in route_tc.cu on tcgen05) -- the router
 // product on the tensor cores (mma.sync) with the fp32 weights split into
 // three bf16 parts.  fp32 tokens or given logits: one CTA per (task, tile of
 // TOK tokens) on the CUDA cores.  The logits
@@ -433,8 +434,11 @@ int launch_route(const Dims &p, const void *x, const float *w_router, const floa
     int st;
     if (p.bf16 && x != nullptr) {
         const __nv_bfloat16 *xb = (const __nv_bfloat16 *)x;
-        st = p.E <= 32 ? launch_mma_router<4>(p, xb, w_router, bias, logits, idx, gate, s)
-                       : launch_mma_router<8>(p, xb, w_router, bias, logits, idx, gate, s);
+        if (route_tc_enabled() && route_tc_width(p) > 0)
+            st = launch_route_tc(p, xb, w_router, bias, logits, idx, gate, s);
+        else
+            st = p.E <= 32 ? launch_mma_router<4>(p, xb, w_router, bias, logits, idx, gate, s)
+                           : launch_mma_router<8>(p, xb, w_router, bias, logits, idx, gate, s);
     } else if (p.bf16) {  // given logits: no GEMV
         st = launch_topk<__nv_bfloat16, 64>(p, nullptr, w_router, bias, logits, idx, gate, s);
     } else {
