@@ -165,7 +165,7 @@ struct PairShape {
     static constexpr int A_SLOTS = (int)((REST - STG_BUFS * 32768u) / KB);
     static constexpr uint32_t EPI_BYTES = 8u * STG_BUFS * 4096u;
     static constexpr uint32_t TMEM_COLS = 2 * BN;
-    static constexpr int NUM_BARS = 2 * A_SLOTS + 3 * B_BUFS + 5;
+    static constexpr int NUM_BARS = 2 * A_SLOTS + 3 * B_BUFS * (B_BUFS == 1 ? NKB : 1) + 5;
     static constexpr size_t SMEM_BYTES =
         1024 + (size_t)B_BUFS * B_BUF + (size_t)A_SLOTS * KB + EPI_BYTES + NUM_BARS * 8 + 16;
     static_assert(A_SLOTS >= 2, "A ring too shallow");
@@ -217,12 +217,21 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     // afull: the leader's counts both CTAs' bytes of the slot (the peer's is unused)
     auto bar_afull = [&](int i) { return bar(i); };
     auto bar_aempty = [&](int i) { return bar(AS + i); };
-    auto bar_bfull = [&](int i) { return bar(2 * AS + i); };
-    auto bar_bempty = [&](int i) { return bar(2 * AS + BB + i); };
-    auto bar_bready = [&](int i) { return bar(2 * AS + 2 * BB + i); };
-    auto bar_tfull = [&](int i) { return bar(2 * AS + 3 * BB + i); };
-    auto bar_tempty = [&](int i) { return bar(2 * AS + 3 * BB + 2 + i); };
-    const uint32_t bar_drain = bar(2 * AS + 3 * BB + 4);
+    // B barriers.  Two buffers: one piece per buffer (the whole tile), handed
+    // to the leader by the tail warp once both CTAs' copies landed.  One
+    // buffer: one piece per k-block, each released by the last row tile's
+    // MMAs on it, so that the next unit's B streams in piece by piece behind
+    // that row tile; dense pieces complete on the leader's barrier, like A,
+    // and need no hand-over.
+    constexpr bool PIECES = BB == 1;
+    constexpr int NPC = PIECES ? NKB : 1;  // B pieces per buffer
+    constexpr int BP = BB * NPC;
+    auto bar_bfull = [&](int bb, int pc) { return bar(2 * AS + bb * NPC + pc); };
+    auto bar_bempty = [&](int bb, int pc) { return bar(2 * AS + BP + bb * NPC + pc); };
+    auto bar_bready = [&](int bb, int pc) { return bar(2 * AS + 2 * BP + bb * NPC + pc); };
+    auto bar_tfull = [&](int i) { return bar(2 * AS + 3 * BP + i); };
+    auto bar_tempty = [&](int i) { return bar(2 * AS + 3 * BP + 2 + i); };
+    const uint32_t bar_drain = bar(2 * AS + 3 * BP + 4);
     volatile int *abort_flag = misc + 1;
     // the peer's abort flag, raised when this CTA gives up
     const uint32_t peer_abort = mapa_shared(smem_u32(misc + 1), rank ^ 1u);
@@ -232,11 +241,12 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             mbar_init(bar_afull(i), 1);
             mbar_init(bar_aempty(i), 1);
         }
-        for (int i = 0; i < BB; ++i) {
-            mbar_init(bar_bfull(i), 1);
-            mbar_init(bar_bempty(i), 1);
-            mbar_init(bar_bready(i), 2);
-        }
+        for (int i = 0; i < BB; ++i)
+            for (int pc = 0; pc < NPC; ++pc) {
+                mbar_init(bar_bfull(i, pc), 1);
+                mbar_init(bar_bempty(i, pc), 1);
+                mbar_init(bar_bready(i, pc), 2);
+            }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar_tfull(i), 1);
             mbar_init(bar_tempty(i), 16);
@@ -285,7 +295,8 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
         if (lane == 0) {
             int ub = 0, ka = 0;
             bool ok = true;
-            int b_issued[BB] = {}, a_issued[AS] = {};
+            // uses of each B piece so far (their parity gives the phase)
+            int b_issued[BP] = {}, a_issued[AS] = {};
             for (int u = u_first; u < u_end && ok; u += u_step) {
                 int g, n_blk, L;
                 decode(u, g, n_blk, L);
@@ -294,27 +305,51 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 if (nkb == 0) continue;
                 const int r0 = L - nkb * BK;  // first row of k-block 0 (<= 0)
                 const int bb = ub % BB;
-                if (!wait_phase(bar_bempty(bb), (uint32_t)((ub / BB) & 1) ^ 1u, abort_flag, args.status))
-                    break;
                 const uint32_t bdst = smem_u32(b_res) + bb * S::B_BUF;
-                mbar_expect_tx(bar_bfull(bb), (KSPLIT ? 2u : 1u) * (uint32_t)nkb * S::KB);
                 const int bchunk = n_blk * 4 + (int)rank * 2;
-                for (int kb = 0; kb < nkb; ++kb) {
-                    const int r = r0 + kb * BK;
-                    tma_load_4d(bdst + kb * S::KB, &tmB, bar_bfull(bb), 0, (cmpb ? crow : 0) + r, bchunk,
-                                cmpb ? 0 : g);
-                    if (KSPLIT) {
-                        if (cmpb)
-                            tma_load_4d(bdst + (NKB + kb) * S::KB, &tmB, bar_bfull(bb), 0, crow + L + r,
-                                        bchunk, 0);
-                        else
-                            tma_load_4d(bdst + (NKB + kb) * S::KB, &tmBlo, bar_bfull(bb), 0, r, bchunk, g);
-                    }
-                }
-                ++b_issued[bb];
                 ++ub;
+                // B piece pc = k-blocks [kb0, kb1) (and their residual), once its
+                // previous use has been released by the MMAs
+                auto load_b = [&](int pc, int kb0, int kb1) -> bool {
+                    int &nb = b_issued[bb * NPC + pc];
+                    if (!wait_phase(bar_bempty(bb, pc), (uint32_t)(nb & 1) ^ 1u, abort_flag, args.status))
+                        return false;
+                    ++nb;
+                    const uint32_t fb = bar_bfull(bb, pc);
+                    const uint32_t bytes = (KSPLIT ? 2u : 1u) * (uint32_t)(kb1 - kb0) * S::KB;
+                    const bool on_leader = PIECES && !cmpb;
+                    const uint32_t fbl = mapa_shared(fb, 0);
+                    if (on_leader) {
+                        if (leader) mbar_expect_tx(fb, 2u * bytes);  // both CTAs' halves
+                    } else {
+                        mbar_expect_tx(fb, bytes);
+                    }
+                    for (int kb = kb0; kb < kb1; ++kb) {
+                        const int r = r0 + kb * BK;
+                        const uint32_t d0 = bdst + kb * S::KB, d1 = bdst + (NKB + kb) * S::KB;
+                        if (cmpb) {
+                            tma_load_4d(d0, &tmB, fb, 0, crow + r, bchunk, 0);
+                            if (KSPLIT) tma_load_4d(d1, &tmB, fb, 0, crow + L + r, bchunk, 0);
+                        } else if (on_leader) {
+                            tma_load_4d_pair(d0, &tmB, fbl, 0, r, bchunk, g);
+                            if (KSPLIT) tma_load_4d_pair(d1, &tmBlo, fbl, 0, r, bchunk, g);
+                        } else {
+                            tma_load_4d(d0, &tmB, fb, 0, r, bchunk, g);
+                            if (KSPLIT) tma_load_4d(d1, &tmBlo, fb, 0, r, bchunk, g);
+                        }
+                    }
+                    return true;
+                };
+                // Two buffers: the whole tile at once (its buffer was freed a
+                // unit ago).  One: each piece just before the first row tile's
+                // A k-block that needs it.
+                if (!PIECES) ok = load_b(0, 0, nkb);
                 for (int m = 0; m < tiles_m && ok; ++m)
                     for (int kb = 0; kb < nkb; ++kb, ++ka) {
+                        if (PIECES && m == 0 && !load_b(kb, kb, kb + 1)) {
+                            ok = false;
+                            break;
+                        }
                         const int sl = ka % AS;
                         if (!wait_phase(bar_aempty(sl), (uint32_t)((ka / AS) & 1) ^ 1u, abort_flag,
                                         args.status)) {
@@ -329,11 +364,13 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             }
             if (*abort_flag) {  // let copies in flight land before the CTA exits
                 const unsigned long long t0 = global_ns();
-                for (int i = 0; i < BB; ++i)
-                    if (b_issued[i] > 0)
-                        while (!mbar_try_wait(bar_bfull(i), (uint32_t)((b_issued[i] - 1) & 1)) &&
-                               global_ns() - t0 < 100000000ull) {
-                        }
+                // (dense B pieces, like A, complete on the leader's barriers)
+                if (leader || !PIECES || cmpb)
+                    for (int i = 0; i < BP; ++i)
+                        if (b_issued[i] > 0)
+                            while (!mbar_try_wait(bar_bfull(i / NPC, i % NPC), (uint32_t)((b_issued[i] - 1) & 1)) &&
+                                   global_ns() - t0 < 100000000ull) {
+                            }
                 // the leader's afull counts the peer's copies too; the peer waits
                 // for the leader at the closing cluster barrier
                 if (leader)
@@ -349,6 +386,7 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
     } else if (warp == 1) {
         // ------------------------------------------------------------ B hand-over (+ MMA in the leader)
         int ub = 0, ka = 0, it = 0;
+        int b_used[BP] = {};  // uses of each B piece so far (their parity gives the phase)
         bool ok = true;
         for (int u = u_first; u < u_end && ok; u += u_step) {
             int g, n_blk, L;
@@ -358,37 +396,52 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
             const int z = nkb * BK - L;  // leading rows of k-block 0 outside the group
             const int skip = z >> 4;     // all-zero 16-row steps of k-block 0
             const int bb = ub % BB;
-            const uint32_t bph = (uint32_t)((ub / BB) & 1);
             uint8_t *bres = b_res + bb * S::B_BUF;
-            if (!wait_phase(bar_bfull(bb), bph, abort_flag, args.status)) break;
-            if (cmpb && z > 0) {
-                // compact B: rows [0, z) of k-block 0 (both parts) hold the
-                // neighbouring entry's rows; zero them (two 64-wide chunks each)
-                for (int part = 0; part < (KSPLIT ? 2 : 1); ++part) {
-                    uint8_t *tile = bres + part * NKB * S::KB;
-                    for (int i = lane; i < 2 * z * 8; i += 32) {
-                        const int c = i / (z * 8), w = i - c * z * 8;
-                        *reinterpret_cast<uint4 *>(tile + c * (BK * 128) + (w >> 3) * 128 + (w & 7) * 16) =
-                            make_uint4(0, 0, 0, 0);
+            ++ub;
+            // Piece pc of this unit's B: wait for this CTA's copy, zero the
+            // compact-B rows of k-block 0 that belong to a neighbour, hand it
+            // to the leader; the leader waits until both CTAs have.
+            auto hand_over = [&](int pc) -> bool {
+                const uint32_t ph = (uint32_t)(b_used[bb * NPC + pc] & 1);
+                ++b_used[bb * NPC + pc];
+                if (!wait_phase(bar_bfull(bb, pc), ph, abort_flag, args.status)) return false;
+                if (cmpb && pc == 0 && z > 0) {
+                    // compact B: rows [0, z) of k-block 0 (both parts) hold the
+                    // neighbouring entry's rows; zero them (two 64-wide chunks each)
+                    for (int part = 0; part < (KSPLIT ? 2 : 1); ++part) {
+                        uint8_t *tile = bres + part * NKB * S::KB;
+                        for (int i = lane; i < 2 * z * 8; i += 32) {
+                            const int c = i / (z * 8), w = i - c * z * 8;
+                            *reinterpret_cast<uint4 *>(tile + c * (BK * 128) + (w >> 3) * 128 + (w & 7) * 16) =
+                                make_uint4(0, 0, 0, 0);
+                        }
                     }
+                    fence_proxy_async();
                 }
-                fence_proxy_async();
-            }
-            __syncwarp();
-            if (lane == 0) mbar_arrive_cluster(mapa_shared(bar_bready(bb), 0));
-            if (!leader) {
-                ++ub;
-                continue;
-            }
-            if (!wait_phase_cluster(bar_bready(bb), bph, abort_flag, args.status)) break;
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(mapa_shared(bar_bready(bb, pc), 0));
+                return !leader || wait_phase_cluster(bar_bready(bb, pc), ph, abort_flag, args.status);
+            };
+            if (!PIECES || cmpb)
+                for (int pc = 0; pc < (PIECES ? nkb : 1) && ok; ++pc) ok = hand_over(pc);
+            if (!leader || !ok) continue;
             for (int m = 0; m < tiles_m && ok; ++m, ++it) {
                 const int acc = it & 1;
+                const bool last_m = m == tiles_m - 1;
                 if (!wait_phase(bar_tempty(acc), (uint32_t)((it >> 1) & 1) ^ 1u, abort_flag, args.status)) {
                     ok = false;
                     break;
                 }
                 tc_fence_after();
                 for (int kb = 0; kb < nkb; ++kb, ++ka) {
+                    if (PIECES && !cmpb && m == 0) {  // dense B piece kb: both halves landed
+                        const uint32_t ph = (uint32_t)(b_used[bb * NPC + kb] & 1);
+                        ++b_used[bb * NPC + kb];
+                        if (!wait_phase(bar_bfull(bb, kb), ph, abort_flag, args.status)) {
+                            ok = false;
+                            break;
+                        }
+                    }
                     const int sl = ka % AS;
                     if (!wait_phase(bar_afull(sl), (uint32_t)((ka / AS) & 1), abort_flag, args.status)) {
                         ok = false;
@@ -407,6 +460,8 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                                               IDESC, (kb | part | (kk - k0)) != 0 ? 1u : 0u);
                         }
                         mma_pair_commit_both(bar_aempty(sl));
+                        // the last row tile's MMAs on a piece are its last use
+                        if (PIECES && last_m) mma_pair_commit_both(bar_bempty(bb, kb));
                     }
                     __syncwarp();
                 }
@@ -415,9 +470,8 @@ wgrad_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant
                 __syncwarp();
             }
             if (!ok) break;
-            if (lane == 0) mma_pair_commit_both(bar_bempty(bb));  // B may be replaced after these MMAs
+            if (!PIECES && lane == 0) mma_pair_commit_both(bar_bempty(bb, 0));  // B may be replaced now
             __syncwarp();
-            ++ub;
         }
         if (leader && lane == 0) {  // all MMAs of the pair complete before TMEM is freed
             mma_pair_commit_local(bar_drain);

@@ -72,8 +72,23 @@ def _zero_pad(t, valid):
                                          ("bf16", 256, 512, 32), ("bf16", 384, 640, 256),
                                          ("f32", 40, 72, 128)])
 def test_group_tails(dtype, d, f, C):
+    _check_tails(dtype, d, f, C, LOADS_BY_C[C])
+
+
+# More groups than SM pairs at C 256, so that each pair takes several units in a
+# row: the SM-pair dW1 kernel's single resident B tile is then released and
+# refilled one k-block at a time while the previous unit's last row tile still
+# runs (d 512: two row tiles per unit; d 256: one).
+@pytest.mark.parametrize("d,f,G", [(512, 512, 96), (256, 768, 160)])
+def test_wgrad_pair_units_in_a_row(d, f, G):
+    rng = np.random.default_rng(7 + d)
+    loads = [int(v) for v in rng.integers(0, 257, size=G)]
+    loads[:4] = [0, 256, 129, 1]  # group 0 empty: its dW must be zeros
+    _check_tails("bf16", d, f, 256, loads)
+
+
+def _check_tails(dtype, d, f, C, loads):
     import paper_2608_16188_gb300 as vm
-    loads = LOADS_BY_C[C]
     G = len(loads)
     p = vm.problem(1, C, d, f, G, 1, 1.0, dtype, capacity=C)
     assert vm.vmoe_problem_capacity(p) == C
