@@ -151,14 +151,17 @@ __device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
 //   dW1, C <= 128 (KSPLIT, NKB 2): B 2 x 64 KB, A 4 slots, staging 32 KB
 //   dW1, C <= 256 (KSPLIT, NKB 4): B 1 x 128 KB, A 4 slots, staging 32 KB
 //   dW2, C <= 128 (NKB 2):         B 2 x 32 KB, A 6 slots, staging 2 x 32 KB
-//   dW2, C <= 256 (NKB 4):         B 2 x 64 KB, A 4 slots, staging 32 KB
+//   dW2, C <= 256 (NKB 4):         B 1 x 64 KB, A 6 slots, staging 2 x 32 KB
 template <bool KSPLIT, int NKB>
 struct PairShape {
     static constexpr int MP = 256;                  // tile rows (MMA M), 128 per CTA
     static constexpr int BN = 256;                  // tile columns (MMA N), 128 per CTA
     static constexpr uint32_t KB = 64 * 128 * 2;    // one k-block of one operand half
     static constexpr uint32_t B_BUF = (KSPLIT ? 2u : 1u) * NKB * KB;
-    static constexpr int B_BUFS = B_BUF <= 65536u ? 2 : 1;
+    // two B buffers for tiles of at most 128 K rows; a tile of more rows is
+    // held once and refilled piece by piece (its shared memory goes to a
+    // double-buffered epilogue staging where it fits)
+    static constexpr int B_BUFS = (B_BUF <= 65536u && NKB <= 2) ? 2 : 1;
     static constexpr uint32_t BUDGET = 224u * 1024u;
     static constexpr uint32_t REST = BUDGET - B_BUFS * B_BUF;
     static constexpr int STG_BUFS = REST >= 160u * 1024u ? 2 : 1;
