@@ -627,12 +627,25 @@ def run_ours(args, cfg, rank, world, local_rank):
             vm.vmoe_expert_bwd_static_scratch(*bw_args)
         torch.cuda.synchronize(dev)
         bw_calls = 10
-        vm.vmoe_trace_enable(bw_calls * 64 + 16)
+        # wall time per call without the kernel trace (its events between
+        # launches would break the programmatic-dependent-launch chain) ...
         t0 = time.perf_counter()
         for _ in range(bw_calls):
             vm.vmoe_expert_bwd_static_scratch(*bw_args)
         torch.cuda.synchronize(dev)
         bw_wall = (time.perf_counter() - t0) / bw_calls
+        # ... the full-workspace backward timed the same way, one call at a time
+        full_args = bw_args + (b.workspace,)
+        t0 = time.perf_counter()
+        for _ in range(bw_calls):
+            vm.vmoe_expert_bwd(*full_args)
+            torch.cuda.synchronize(dev)
+        full_wall = (time.perf_counter() - t0) / bw_calls
+        # ... and the kernels' device times from a traced pass
+        vm.vmoe_trace_enable(bw_calls * 64 + 16)
+        for _ in range(bw_calls):
+            vm.vmoe_expert_bwd_static_scratch(*bw_args)
+        torch.cuda.synchronize(dev)
         n_bw = vm.vmoe_trace_disable()
         bw_kernel_ms = sum(vm.vmoe_trace_get(i)[1] for i in range(n_bw)) / bw_calls
         st = vm.vmoe_device_status()
@@ -718,6 +731,7 @@ def run_ours(args, cfg, rank, world, local_rank):
             "budget_bytes": vm.VMOE_STATIC_SCRATCH_BYTES,
             "full_workspace_bytes": vm.vmoe_expert_bwd_workspace_size(p),
             "ms_per_call_wall": round(bw_wall * 1e3, 4),
+            "full_workspace_ms_per_call_wall": round(full_wall * 1e3, 4),
             "kernel_ms_per_call": round(bw_kernel_ms, 4),
             "launches_per_call": n_bw // bw_calls,
             "full_workspace_kernel_ms": round(sum(kstats[k]["ms_avg"] for k in

@@ -6,11 +6,10 @@
 #include <vector>
 
 #include "gemm_tc2.cuh"
+#include "planner.cuh"
 
 namespace vmoe {
 
-int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
-                double budget, int32_t *order, int32_t *slice_start);  // planner.cu
 int plan_shares(int n, const double *work, const int32_t *minimum, const int32_t *saturation,
                 int32_t budget, int32_t *shares);                      // planner.cu
 
@@ -83,9 +82,14 @@ int launch_expert_bwd_bf16(const Dims &p, const __nv_bfloat16 *xe, const __nv_bf
 // its dH rows (load rows of dH_hi, then load rows of the residual), in units of
 // BW_UNIT rows; the slice's groups are packed into the workspace at 8-row
 // offsets, and dA, dX and dW1 run per slice.  dW2 needs no dH and runs once.
-// The loads are read back to the host first (one stream synchronisation); the
-// plan (group list and first rows) goes to the head of the workspace.
+// The loads are read back to the host first (one stream synchronisation).
+// dW2 is launched before any planning, and the DP hands out one slice at a
+// time: the host places the groups of slice s + 1 while the GPU runs slice s
+// (and, for the first slice, dW2).  Each slice's plan (group list and first
+// rows) reaches the head of the workspace through a small kernel whose
+// parameters carry it, so no host copy waits for the stream.
 constexpr int BW_UNIT = 8;
+constexpr int PLAN_CHUNK = 256;
 
 size_t bwd_plan_bytes(const Dims &p) { return (((size_t)2 * p.G() * sizeof(int32_t)) + 255) & ~(size_t)255; }
 
@@ -93,6 +97,25 @@ size_t bwd_min_workspace(const Dims &p) {
     const size_t unit_rows = ((size_t)2 * p.C + BW_UNIT - 1) / BW_UNIT * BW_UNIT;
     return bwd_plan_bytes(p) + unit_rows * p.f * sizeof(__nv_bfloat16);
 }
+
+namespace {
+// Up to PLAN_CHUNK plan entries of one slice, by value: entry pos + i is group
+// g[i], whose dH rows start at row[i] of the workspace.
+struct PlanChunk {
+    int32_t n, pos, G;
+    int32_t g[PLAN_CHUNK];
+    int32_t row[PLAN_CHUNK];
+};
+
+__global__ void __launch_bounds__(PLAN_CHUNK) plan_write_kernel(const __grid_constant__ PlanChunk c,
+                                                               int32_t *__restrict__ plan) {
+    const int i = threadIdx.x;
+    if (i < c.n) {
+        plan[c.pos + i] = c.g[i];
+        plan[c.G + c.pos + i] = c.row[i];
+    }
+}
+}  // namespace
 
 int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const __nv_bfloat16 *h,
                                   const __nv_bfloat16 *act, const __nv_bfloat16 *w1,
@@ -123,25 +146,13 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
     // no slice needs more than every group's footprint: that bounds the DP table
     long long cap_units = rows / BW_UNIT;
     if (cap_units > total_units) cap_units = total_units;
-    std::vector<int32_t> order(G), start(G + 1);
-    const int ns = plan_slices(G, w.data(), r.data(), cap_units, 0.0, 0.0, order.data(), start.data());
-    if (ns < 0) return ns;
-    // plan on the device: [glist (G)][crow (G)], slice by slice
-    std::vector<int32_t> plan(2 * (size_t)G);
-    for (int sidx = 0; sidx < ns; ++sidx) {
-        long long row = 0;
-        for (int k = start[sidx]; k < start[sidx + 1]; ++k) {
-            plan[k] = order[k];
-            plan[G + k] = (int32_t)row;
-            row += w[order[k]] * BW_UNIT;
-        }
-    }
+    SlicePlanner planner;
+    int st = planner.init(G, w.data(), r.data(), cap_units, 0.0, 0.0);
+    if (st != VMOE_OK) return st;
+    // dW2 first: it needs no dH, and it runs while the first slice is planned
+    if ((st = wgrad_gemm(p, act, p.f, dye, p.d, load, dw2, s, "tc_dw2")) != VMOE_OK) return st;
     int32_t *dplan = reinterpret_cast<int32_t *>(workspace);
     __nv_bfloat16 *dh = reinterpret_cast<__nv_bfloat16 *>(static_cast<uint8_t *>(workspace) + plan_bytes);
-    if (cudaMemcpyAsync(dplan, plan.data(), sizeof(int32_t) * 2 * G, cudaMemcpyHostToDevice, s) !=
-        cudaSuccess)
-        return VMOE_ERR_CUDA;
-    if (cudaStreamSynchronize(s) != cudaSuccess) return VMOE_ERR_CUDA;  // host plan buffer is freed on return
     // dW1 of a slice on SM pairs, optionally (VMOE_SHARES=1) with each group's
     // column tiles on a share of the pairs from the fill-clamp-refill allocation
     // (Section 3.2.2): work = its tiles x (output bytes + load x input bytes per
@@ -150,15 +161,15 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
     const bool use_shares = shares_enabled() && pair_enabled() && p.d % 256 == 0 && p.f % 256 == 0 &&
                             p.C <= 4 * BK;
     const int pairs = use_shares ? pair_wgrad_capacity<true>(p.C) : 0;
-    auto slice_schedule = [&](int sidx, PairSchedule &sc) {
+    auto slice_schedule = [&](const std::vector<int> &slice, PairSchedule &sc) {
         sc.enabled = 0;
-        const int n = start[sidx + 1] - start[sidx];
+        const int n = (int)slice.size();
         if (pairs <= 0 || n > pairs || pairs > MAX_PAIRS) return;
         const int units = p.f / 256, tiles_m = p.d / 256;
         std::vector<double> work(n);
         std::vector<int32_t> mn(n, 1), sat(n, units), share(n);
         for (int i = 0; i < n; ++i) {
-            const double L = hload[order[start[sidx] + i]];
+            const double L = hload[slice[i]];
             work[i] = units * ((double)tiles_m * 256 * 256 * 2 + L * ((double)p.d * 2 + 4 * 256));
         }
         if (plan_shares(n, work.data(), mn.data(), sat.data(), pairs, share.data()) < 0) return;
@@ -172,12 +183,32 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
         for (; c < MAX_PAIRS; ++c) sc.first[c] = sc.count[c] = 0;
         sc.enabled = 1;
     };
-    int st = VMOE_OK;
-    for (int sidx = 0; sidx < ns && st == VMOE_OK; ++sidx) {
+    std::vector<int> slice;
+    int pos = 0, ns = 0;
+    while (st == VMOE_OK && planner.next(slice)) {
+        const int n = (int)slice.size();
+        // this slice's plan entries [pos, pos + n) on the device
+        PlanChunk c;
+        c.G = G;
+        long long row = 0;
+        for (int k0 = 0; k0 < n && st == VMOE_OK; k0 += PLAN_CHUNK) {
+            c.pos = pos + k0;
+            c.n = n - k0 < PLAN_CHUNK ? n - k0 : PLAN_CHUNK;
+            for (int i = 0; i < c.n; ++i) {
+                c.g[i] = slice[k0 + i];
+                c.row[i] = (int32_t)row;
+                row += w[slice[k0 + i]] * BW_UNIT;
+            }
+            trace_before(s, "bwd_plan");
+            plan_write_kernel<<<1, PLAN_CHUNK, 0, s>>>(c, dplan);
+            st = launch_result();
+            trace_after(s);
+        }
+        if (st != VMOE_OK) break;
         Slice sl;
-        sl.glist = dplan + start[sidx];
-        sl.crow = dplan + G + start[sidx];
-        sl.n = start[sidx + 1] - start[sidx];
+        sl.glist = dplan + pos;
+        sl.crow = dplan + G + pos;
+        sl.n = n;
         sl.rows = rows;
         sl.compact = CMP_D;
         st = row_gemm<EPI_DGELU, false>(p, dye, p.d, w2, p.f, load, dh, dh, h, s, "tc_da_dgelu", 0, 0, 0,
@@ -189,10 +220,11 @@ int launch_expert_bwd_bf16_sliced(const Dims &p, const __nv_bfloat16 *xe, const 
         if (st != VMOE_OK) break;
         sl.compact = CMP_B;
         PairSchedule sc;
-        slice_schedule(sidx, sc);
+        slice_schedule(slice, sc);
         st = wgrad_gemm(p, xe, p.d, dh, p.f, load, dw1, s, "tc_dw1", true, sl, &sc);
+        pos += n;
+        ++ns;
     }
-    if (st == VMOE_OK) st = wgrad_gemm(p, act, p.f, dye, p.d, load, dw2, s, "tc_dw2");
     if (nslices_out) *nslices_out = ns;
     return st;
 }

@@ -22,84 +22,105 @@
 #include <numeric>
 #include <vector>
 
+#include "planner.cuh"
 #include "vmoe.h"
 
 namespace vmoe {
 
-int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
-                double budget, int32_t *order, int32_t *slice_start) {
-    if (n < 0 || capacity < 0 || (n > 0 && (!weight || !lifespan || !order || !slice_start)))
-        return VMOE_ERR_INVALID;
-    if (!slice_start) return VMOE_ERR_INVALID;
+int SlicePlanner::init(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
+                       double budget) {
+    if (n < 0 || capacity < 0 || (n > 0 && (!weight || !lifespan))) return VMOE_ERR_INVALID;
     for (int i = 0; i < n; ++i) {
         if (weight[i] < 0 || !(lifespan[i] == lifespan[i])) return VMOE_ERR_INVALID;
         if (weight[i] > capacity) return VMOE_ERR_UNSUPPORTED;
     }
     if (capacity >= (1 << 24) || (int64_t)n * (capacity + 1) > ((int64_t)1 << 30))
         return VMOE_ERR_UNSUPPORTED;  // DP table too large
-    const int cap = (int)capacity;
+    weight_ = weight;
+    n_ = n;
+    cap_ = (int)capacity;
+    first_ = true;
     const double mc = budget > 0.0 ? budget : (double)capacity;
-    std::vector<double> v(n);
-    for (int i = 0; i < n; ++i) v[i] = (mc > 0.0 ? (double)weight[i] / mc : 0.0) - eta * lifespan[i];
+    v_.assign(n, 0.0);
+    for (int i = 0; i < n; ++i) v_[i] = (mc > 0.0 ? (double)weight[i] / mc : 0.0) - eta * lifespan[i];
     std::vector<int> sjf(n);
     std::iota(sjf.begin(), sjf.end(), 0);
     std::stable_sort(sjf.begin(), sjf.end(), [&](int a, int b) { return lifespan[a] < lifespan[b]; });
-    std::vector<int> zero, remaining;
-    for (int i : sjf) (weight[i] == 0 ? zero : remaining).push_back(i);
-
-    std::vector<std::vector<int>> slices;
+    zero_.clear();
+    remaining_.clear();
+    for (int i : sjf) (weight[i] == 0 ? zero_ : remaining_).push_back(i);
     // Two DP rows, row a-1 (cur) -> row a (nxt): every entry of row a depends on
     // row a-1 only, so the update is branch-free and vectorises; the decision
     // table gets every entry written, so it needs no clearing.
-    std::vector<double> cur(cap + 1), nxt(cap + 1);
-    std::unique_ptr<uint8_t[]> take(new uint8_t[(size_t)n * (cap + 1)]);
-    while (!remaining.empty()) {
-        const int m = (int)remaining.size();
-        std::fill(cur.begin(), cur.end(), 0.0);
-        for (int a = 0; a < m; ++a) {
-            const int i = remaining[a];
-            const int wi = (int)weight[i];
-            const double vi = v[i];
-            uint8_t *__restrict__ t = take.get() + (size_t)a * (cap + 1);
-            const double *__restrict__ o = cur.data();
-            double *__restrict__ nw = nxt.data();
-            for (int j = 0; j < wi; ++j) {
-                nw[j] = o[j];
-                t[j] = 0;
-            }
-            for (int j = wi; j <= cap; ++j) {  // taken only when strictly better
-                const double cand = o[j - wi] + vi;
-                const bool tk = cand > o[j];
-                nw[j] = tk ? cand : o[j];
-                t[j] = tk;
-            }
-            cur.swap(nxt);
+    cur_.assign(cap_ + 1, 0.0);
+    nxt_.assign(cap_ + 1, 0.0);
+    chosen_.assign(n, 0);
+    take_.reset(new uint8_t[(size_t)(remaining_.size() > 0 ? remaining_.size() : 1) * (cap_ + 1)]);
+    return VMOE_OK;
+}
+
+bool SlicePlanner::next(std::vector<int> &slice) {
+    slice.clear();
+    const bool first = first_;
+    first_ = false;
+    if (first) slice = zero_;  // zero-footprint experts join the first slice
+    if (remaining_.empty()) return first && n_ > 0;
+    const int m = (int)remaining_.size(), cap = cap_;
+    std::fill(cur_.begin(), cur_.end(), 0.0);
+    for (int a = 0; a < m; ++a) {
+        const int i = remaining_[a];
+        const int wi = (int)weight_[i];
+        const double vi = v_[i];
+        uint8_t *__restrict__ t = take_.get() + (size_t)a * (cap + 1);
+        const double *__restrict__ o = cur_.data();
+        double *__restrict__ nw = nxt_.data();
+        for (int j = 0; j < wi; ++j) {
+            nw[j] = o[j];
+            t[j] = 0;
         }
-        std::vector<uint8_t> chosen(n, 0);
-        int nchosen = 0;
-        for (int a = m - 1, j = cap; a >= 0; --a)
-            if (take[(size_t)a * (cap + 1) + j]) {
-                chosen[remaining[a]] = 1;
-                ++nchosen;
-                j -= (int)weight[remaining[a]];
-            }
-        if (nchosen == 0) chosen[remaining[0]] = 1;
-        std::vector<int> slice, rest;
-        for (int i : remaining) (chosen[i] ? slice : rest).push_back(i);
-        slices.push_back(std::move(slice));
-        remaining.swap(rest);
+        for (int j = wi; j <= cap; ++j) {  // taken only when strictly better
+            const double cand = o[j - wi] + vi;
+            const bool tk = cand > o[j];
+            nw[j] = tk ? cand : o[j];
+            t[j] = tk;
+        }
+        cur_.swap(nxt_);
     }
-    if (!zero.empty()) {
-        if (slices.empty()) slices.push_back({});
-        slices[0].insert(slices[0].begin(), zero.begin(), zero.end());
+    int nchosen = 0;
+    for (int a = m - 1, j = cap; a >= 0; --a)
+        if (take_[(size_t)a * (cap + 1) + j]) {
+            chosen_[remaining_[a]] = 1;
+            ++nchosen;
+            j -= (int)weight_[remaining_[a]];
+        }
+    if (nchosen == 0) chosen_[remaining_[0]] = 1;  // an empty choice: the first expert alone
+    std::vector<int> rest;
+    for (int i : remaining_) {
+        if (chosen_[i]) {
+            slice.push_back(i);
+            chosen_[i] = 0;
+        } else {
+            rest.push_back(i);
+        }
     }
-    int pos = 0;
-    for (size_t s = 0; s < slices.size(); ++s) {
-        slice_start[s] = pos;
-        for (int i : slices[s]) order[pos++] = i;
+    remaining_.swap(rest);
+    return true;
+}
+
+int plan_slices(int n, const int64_t *weight, const double *lifespan, int64_t capacity, double eta,
+                double budget, int32_t *order, int32_t *slice_start) {
+    if (n < 0 || (n > 0 && !order) || !slice_start) return VMOE_ERR_INVALID;
+    SlicePlanner planner;
+    const int st = planner.init(n, weight, lifespan, capacity, eta, budget);
+    if (st != VMOE_OK) return st;
+    std::vector<int> slice;
+    int pos = 0, ns = 0;
+    while (planner.next(slice)) {
+        slice_start[ns++] = pos;
+        for (int i : slice) order[pos++] = i;
     }
-    slice_start[slices.size()] = pos;
-    return (int)slices.size();
+    slice_start[ns] = pos;
+    return ns;
 }
 
 // Section 3.2.2 (lifespan-aware aligning): the fill-clamp-refill allocation of a
