@@ -196,7 +196,7 @@ def write_traffic_record(workload, tasks, plain_json, captures, path=None):
                      "bench.py scales them to the full workload by the algorithmic bytes and drops a "
                      "record once the kernel's sources change (sources_sha256).")
     wl = data.setdefault("workloads", {}).setdefault(workload, {})
-    wl["tasks"] = tasks
+    wl.pop("tasks", None)  # per kernel: captured_at_tasks
     kern = wl.setdefault("kernels", {})
     for name, log in captures:
         vals = {}
@@ -211,6 +211,7 @@ def write_traffic_record(workload, tasks, plain_json, captures, path=None):
             continue
         kern[name] = {"dram_bytes_per_launch": int(sum(vals.values())),
                       "algorithmic_bytes_per_launch": int(algo[name]),
+                      "captured_at_tasks": tasks,
                       "source_files": ["paper_2608_16188_gb300/csrc/" + f for f in KERNEL_SOURCES[name]],
                       "sources_sha256": sources_sha256(name)}
     with open(path, "w") as fh:

@@ -178,8 +178,11 @@ size_t vmoe_expert_bwd_min_workspace_size(const vmoe_problem *p);
  *   placed in slices whose dH fits (the cross-task DP of vmoe_plan_slices,
  *   Section 3.2.1, each group's footprint its dH rows, its lifespan its load)
  *   and dA, dX and dW1 run slice by slice.  That path reads `load` back to the
- *   host first and synchronises `cuda_stream`.  The results are bitwise the
- *   same either way.  Less than the minimum, or NULL, returns VMOE_ERR_INVALID. */
+ *   host first and synchronises `cuda_stream` (once); it then launches dW2 and
+ *   plans one slice at a time, each slice's kernels queued as soon as it is
+ *   placed, and returns when the last slice is queued.  The results are
+ *   bitwise the same either way.  Less than the minimum, or NULL, returns
+ *   VMOE_ERR_INVALID. */
 int vmoe_expert_bwd(const vmoe_problem *p, const void *xe, const void *h, const void *a,
                     const void *w1, const void *w2, const void *dye, const int32_t *load,
                     void *dxe, void *dw1, void *dw2, void *workspace, size_t workspace_bytes,

@@ -54,7 +54,8 @@ def test_write_traffic_record_round_trip(tmp_path):
     out = tmp_path / "rec.json"
     bench.write_traffic_record("vitb_t17", 2, str(plain), [("tc_dw1", str(log))], path=str(out))
     rec = json.loads(out.read_text())["workloads"]["vitb_t17"]
-    assert rec["tasks"] == 2 and rec["kernels"]["tc_dw1"]["dram_bytes_per_launch"] == 1500500
+    assert rec["kernels"]["tc_dw1"]["captured_at_tasks"] == 2
+    assert rec["kernels"]["tc_dw1"]["dram_bytes_per_launch"] == 1500500
     assert bench.traffic_record("tc_dw1", "vitb_t17", 2000, str(out)) == 3001000.0
 
 
@@ -63,9 +64,10 @@ def test_committed_record_names_known_workloads_and_kernels():
         rec = json.load(fh)
     for wl, entry in rec["workloads"].items():
         assert wl in bench.workloads.CONFIGS
-        assert entry["tasks"] < bench.workloads.CONFIGS[wl].T  # a prefix, not the full size
-        for name in entry["kernels"]:
+        for name, k in entry["kernels"].items():
             assert name in bench.KERNEL_SOURCES
+            # a prefix of the tasks, or the full size (one-pass DRAM counters only)
+            assert 1 <= k["captured_at_tasks"] <= bench.workloads.CONFIGS[wl].T
 
 
 def test_l2_policy():
