@@ -4,7 +4,8 @@ cross-task DP (Section 3.2.1) and dA, dX and dW1 address a compact dH buffer.
 Every group's GEMMs are the same as in the unsliced run, so dXe (valid rows), dW1
 and dW2 must be bitwise equal to it -- at the smallest workspace (about one group
 per slice), at a third of the full size, for groups of two row tiles (the
-streaming weight-gradient kernel), with empty groups, and with 512 groups.
+streaming weight-gradient kernel), with empty groups, with 512 groups, and with
+1024 groups whose first slice holds more than 256 entries.
 """
 import pytest
 import torch
@@ -24,6 +25,10 @@ CASES = {
                           dtype="bf16", bias="drift"),
     "512_groups": Config("sl_512", 83, T=2, N=300, d=128, f=128, E=256, k=8, cf=2.0,
                          dtype="bf16", bias="drift"),
+    # 1024 groups, most of them empty: the empty groups join the first slice, so
+    # its plan (more than 256 entries) reaches the device in several parts
+    "1024_groups_mostly_empty": Config("sl_1024", 84, T=4, N=64, d=128, f=128, E=256, k=2,
+                                       cf=2.0, dtype="bf16", bias="drift"),
 }
 
 
