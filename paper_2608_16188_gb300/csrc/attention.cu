@@ -19,6 +19,8 @@
 // shared memory -- a group holds at most C <= 512 tokens -- so the softmax of a
 // row runs online over key blocks of 64 with the row maximum subtracted, and
 // the forward saves each row's log-sum-exp for the backward to rebuild P.
+// The tiles arrive by cp.async, one commit group per block of 64 keys (or
+// queries), so the work on block j overlaps the copies of the blocks after it.
 // Keys (or queries) past the load are masked; rows past it are never stored.
 // There are no atomics: dQ is one kernel over query blocks, dK and dV another
 // over key blocks, so every sum runs in a fixed order.
@@ -73,15 +75,37 @@ __device__ __forceinline__ int clamp_load(const int32_t *load, int g, int C) {
 }
 
 // Rows [r0, r0 + n) of the 64 columns at `col` of a [C][ld] bf16 matrix of group
-// g into a shared tile [n][AT_PITCH]; rows at or past `valid` are zero.
-__device__ __forceinline__ void at_load_rows(__nv_bfloat16 *dst, const __nv_bfloat16 *src, int ld, int r0,
-                                             int n, int valid, int col) {
+// g into a shared tile [n][AT_PITCH], rows at or past `valid` zero, by cp.async
+// (16-byte copies straight to shared memory, zero-filled past `valid`; an
+// invalid row's source address is clamped to row 0, which is not read), in the
+// commit group the caller closes.
+__device__ __forceinline__ void at_cp_rows(__nv_bfloat16 *dst, const __nv_bfloat16 *src, int ld, int r0, int n,
+                                           int valid, int col) {
     for (int i = threadIdx.x; i < n * 8; i += AT_THREADS) {
         const int r = i >> 3, c8 = (i & 7) * 8;
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (r0 + r < valid) v = __ldg(reinterpret_cast<const uint4 *>(src + (long long)(r0 + r) * ld + col + c8));
-        *reinterpret_cast<uint4 *>(dst + r * AT_PITCH + c8) = v;
+        const bool ok = r0 + r < valid;
+        const __nv_bfloat16 *g = src + (long long)(ok ? r0 + r : 0) * ld + col + c8;
+        const uint32_t d = (uint32_t)__cvta_generic_to_shared(dst + r * AT_PITCH + c8);
+        asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(g), "r"(ok ? 16 : 0)
+                     : "memory");
     }
+}
+__device__ __forceinline__ void at_cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+// Waits until at most `pending` of this thread's newest commit groups are still
+// in flight (0..7: a group holds at most 8 key or query blocks), then makes
+// every thread's landed copies visible to the CTA.
+__device__ __forceinline__ void at_cp_wait(int pending) {
+    switch (pending) {
+        case 0: asm volatile("cp.async.wait_group 0;\n" ::: "memory"); break;
+        case 1: asm volatile("cp.async.wait_group 1;\n" ::: "memory"); break;
+        case 2: asm volatile("cp.async.wait_group 2;\n" ::: "memory"); break;
+        case 3: asm volatile("cp.async.wait_group 3;\n" ::: "memory"); break;
+        case 4: asm volatile("cp.async.wait_group 4;\n" ::: "memory"); break;
+        case 5: asm volatile("cp.async.wait_group 5;\n" ::: "memory"); break;
+        case 6: asm volatile("cp.async.wait_group 6;\n" ::: "memory"); break;
+        default: asm volatile("cp.async.wait_group 7;\n" ::: "memory"); break;
+    }
+    __syncthreads();
 }
 
 // A fragments (16 rows x 64 columns, four k16 steps) of a warp's 16 rows of a
@@ -176,16 +200,22 @@ __global__ void __launch_bounds__(AT_THREADS) attn_fwd_kernel(AtArgs a) {
     extern __shared__ __align__(16) __nv_bfloat16 at_smem[];
     __nv_bfloat16 *qs = at_smem, *ks = qs + AT_BLK * AT_PITCH, *vs = ks + Lp * AT_PITCH;
     const __nv_bfloat16 *src = a.qkv + (long long)g * a.C * ld;
-    at_load_rows(qs, src, ld, q0, AT_BLK, L, h * AT_DK);
-    at_load_rows(ks, src, ld, 0, Lp, L, (H + h) * AT_DK);
-    at_load_rows(vs, src, ld, 0, Lp, L, (2 * H + h) * AT_DK);
-    __syncthreads();
+    // commit group 0: the queries and key block 0; group j: key block j
+    const int nkb = Lp / AT_BLK;
+    at_cp_rows(qs, src, ld, q0, AT_BLK, L, h * AT_DK);
+    for (int j = 0; j < nkb; ++j) {
+        at_cp_rows(ks + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, (H + h) * AT_DK);
+        at_cp_rows(vs + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, (2 * H + h) * AT_DK);
+        at_cp_commit();
+    }
+    at_cp_wait(nkb - 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = lane & 3;
     uint32_t qa[4][4];
     at_afrag(qa, qs, warp * 16);
     float o[8][4], mrow[2] = {-INFINITY, -INFINITY}, lrow[2] = {0.0f, 0.0f};
     at_zero(o);
     for (int kb = 0; kb < Lp; kb += AT_BLK) {
+        if (kb > 0) at_cp_wait(nkb - 1 - kb / AT_BLK);
         float s[8][4];
         at_zero(s);
         at_mma_abt(s, qa, ks, kb);
@@ -251,12 +281,17 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
     float *dsh = reinterpret_cast<float *>(vs + Lp * AT_PITCH);  // [64] D of the block
     const __nv_bfloat16 *src = a.qkv + (long long)g * a.C * ld;
     const long long ob = (long long)g * a.C * ldo;
-    at_load_rows(qs, src, ld, q0, AT_BLK, L, h * AT_DK);
-    at_load_rows(dos, a.dout + ob, ldo, q0, AT_BLK, L, h * AT_DK);
-    at_load_rows(os, a.o + ob, ldo, q0, AT_BLK, L, h * AT_DK);
-    at_load_rows(ks, src, ld, 0, Lp, L, (H + h) * AT_DK);
-    at_load_rows(vs, src, ld, 0, Lp, L, (2 * H + h) * AT_DK);
-    __syncthreads();
+    // commit group 0: this block's Q, dO, O and key block 0; group j: key block j
+    const int nkb = Lp / AT_BLK;
+    at_cp_rows(qs, src, ld, q0, AT_BLK, L, h * AT_DK);
+    at_cp_rows(dos, a.dout + ob, ldo, q0, AT_BLK, L, h * AT_DK);
+    at_cp_rows(os, a.o + ob, ldo, q0, AT_BLK, L, h * AT_DK);
+    for (int j = 0; j < nkb; ++j) {
+        at_cp_rows(ks + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, (H + h) * AT_DK);
+        at_cp_rows(vs + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, (2 * H + h) * AT_DK);
+        at_cp_commit();
+    }
+    at_cp_wait(nkb - 1);
     // D: two threads per row, 32 columns each, in a fixed order
     {
         const int r = threadIdx.x >> 1, c0 = (threadIdx.x & 1) * 32;
@@ -285,6 +320,7 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
     float dq[8][4];
     at_zero(dq);
     for (int kb = 0; kb < Lp; kb += AT_BLK) {
+        if (kb > 0) at_cp_wait(nkb - 1 - kb / AT_BLK);
         float s[8][4], dp[8][4];
         at_zero(s);
         at_zero(dp);
@@ -321,16 +357,21 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dkv_kern
     float *lse_s = reinterpret_cast<float *>(dos + Lp * AT_PITCH), *d_s = lse_s + Lp;
     const __nv_bfloat16 *src = a.qkv + (long long)g * a.C * ld;
     const long long ob = (long long)g * a.C * ldo;
-    at_load_rows(ks, src, ld, k0, AT_BLK, L, (H + h) * AT_DK);
-    at_load_rows(vs, src, ld, k0, AT_BLK, L, (2 * H + h) * AT_DK);
-    at_load_rows(qs, src, ld, 0, Lp, L, h * AT_DK);
-    at_load_rows(dos, a.dout + ob, ldo, 0, Lp, L, h * AT_DK);
+    // commit group 0: this block's K, V and query block 0; group j: query block j
+    const int nqb = Lp / AT_BLK;
+    at_cp_rows(ks, src, ld, k0, AT_BLK, L, (H + h) * AT_DK);
+    at_cp_rows(vs, src, ld, k0, AT_BLK, L, (2 * H + h) * AT_DK);
+    for (int j = 0; j < nqb; ++j) {
+        at_cp_rows(qs + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, h * AT_DK);
+        at_cp_rows(dos + j * AT_BLK * AT_PITCH, a.dout + ob, ldo, j * AT_BLK, AT_BLK, L, h * AT_DK);
+        at_cp_commit();
+    }
     for (int i = threadIdx.x; i < Lp; i += AT_THREADS) {
         const bool v = i < L;
         lse_s[i] = v ? __ldg(a.lse + ((long long)g * H + h) * a.C + i) : 0.0f;
         d_s[i] = v ? __ldg(a.dsum + ((long long)g * H + h) * a.C + i) : 0.0f;
     }
-    __syncthreads();
+    at_cp_wait(nqb - 1);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = lane & 3;
     uint32_t ka[4][4], va[4][4];
     at_afrag(ka, ks, warp * 16);
@@ -339,6 +380,7 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dkv_kern
     at_zero(dk);
     at_zero(dv);
     for (int qb = 0; qb < Lp; qb += AT_BLK) {
+        if (qb > 0) at_cp_wait(nqb - 1 - qb / AT_BLK);
         float st[8][4], dpt[8][4];
         at_zero(st);
         at_zero(dpt);
