@@ -79,9 +79,10 @@ __device__ __forceinline__ int clamp_load(const int32_t *load, int g, int C) {
 // (16-byte copies straight to shared memory, zero-filled past `valid`; an
 // invalid row's source address is clamped to row 0, which is not read), in the
 // commit group the caller closes.
-__device__ __forceinline__ void at_cp_rows(__nv_bfloat16 *dst, const __nv_bfloat16 *src, int ld, int r0, int n,
-                                           int valid, int col) {
-    for (int i = threadIdx.x; i < n * 8; i += AT_THREADS) {
+template <int NTHREADS>
+__device__ __forceinline__ void at_cp_rows_n(__nv_bfloat16 *dst, const __nv_bfloat16 *src, int ld, int r0, int n,
+                                             int valid, int col) {
+    for (int i = threadIdx.x; i < n * 8; i += NTHREADS) {
         const int r = i >> 3, c8 = (i & 7) * 8;
         const bool ok = r0 + r < valid;
         const __nv_bfloat16 *g = src + (long long)(ok ? r0 + r : 0) * ld + col + c8;
@@ -89,6 +90,10 @@ __device__ __forceinline__ void at_cp_rows(__nv_bfloat16 *dst, const __nv_bfloat
         asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(g), "r"(ok ? 16 : 0)
                      : "memory");
     }
+}
+__device__ __forceinline__ void at_cp_rows(__nv_bfloat16 *dst, const __nv_bfloat16 *src, int ld, int r0, int n,
+                                           int valid, int col) {
+    at_cp_rows_n<AT_THREADS>(dst, src, ld, r0, n, valid, col);
 }
 __device__ __forceinline__ void at_cp_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
 // Waits until at most `pending` of this thread's newest commit groups are still
@@ -402,6 +407,146 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dkv_kern
     at_store(dv, 1.0f, dst, ld, k0 + warp * 16, L, (2 * H + h) * AT_DK);
 }
 
+// ------------------------------------------------------------------ backward, groups of <= 128 tokens
+// One CTA of 8 warps per (head, group) with L <= 128: S, P, dP and dS are formed
+// once for all queries and keys instead of in both kernels above.  Warp w owns
+// queries [16 w, 16 w + 16).  Per block of 64 keys: S = Q K^T, dP = dO V^T,
+// P = exp(S / sqrt(dk) - lse), dS = P (dP - D) (zero for queries or keys past
+// L), dQ += dS K in registers; P and dS (bf16, as the MMAs round them) go to
+// shared memory, and warps 0-3 form dV = P^T dO and warps 4-7 dK = dS^T Q for
+// the block's 64 keys (16 a warp), summed over the queries in increasing order.
+constexpr int AF_THREADS = 256;
+constexpr int AF_ROWS = 128;
+
+// acc[8][4] (16 keys x 64) += A^T B: A = 16 key columns (from acol) of a shared
+// [query][key] tile, B = a shared [query][64] tile, over queries [0, nq) in
+// steps of 16 (A fragments by ldmatrix.trans: A's rows are the tile's columns).
+__device__ __forceinline__ void at_mma_tb(float (&acc)[8][4], const __nv_bfloat16 *atile, int acol,
+                                          const __nv_bfloat16 *btile, int nq) {
+    const int lane = threadIdx.x & 31, m = lane >> 3;
+    for (int q0 = 0; q0 < nq; q0 += 16) {
+        uint32_t a[4];
+        at_ldsm_x4_t(a, atile + (q0 + (lane & 7) + (lane >> 4) * 8) * AT_PITCH + acol + (m & 1) * 8);
+#pragma unroll
+        for (int dp = 0; dp < 4; ++dp) {
+            uint32_t b[4];
+            at_ldsm_x4_t(b, btile + (q0 + (m & 1) * 8 + (lane & 7)) * AT_PITCH + dp * 16 + (m >> 1) * 8);
+            mma_bf16_16816(acc[2 * dp], a[0], a[1], a[2], a[3], b[0], b[1]);
+            mma_bf16_16816(acc[2 * dp + 1], a[0], a[1], a[2], a[3], b[2], b[3]);
+        }
+    }
+}
+
+// A warp's 16 x 64 fp32 tile as bf16 into rows row0.. of a shared [rows][AT_PITCH] tile.
+__device__ __forceinline__ void at_put(__nv_bfloat16 *tile, int row0, const float (&v)[8][4]) {
+    const int lane = threadIdx.x & 31, g = lane >> 2, t = lane & 3;
+#pragma unroll
+    for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int nt = 0; nt < 8; ++nt)
+            *reinterpret_cast<uint32_t *>(tile + (row0 + g + 8 * h) * AT_PITCH + nt * 8 + 2 * t) =
+                pack_bf16x2(v[nt][2 * h], v[nt][2 * h + 1]);
+}
+
+__global__ void __launch_bounds__(AF_THREADS, 2) attn_bwd_fused_kernel(AtArgs a) {
+    pdl_wait();
+    const int h = blockIdx.y, g = blockIdx.z;
+    const int L = clamp_load(a.load, g, a.C);
+    if (L == 0) return;
+    const int Lp = (L + AT_BLK - 1) / AT_BLK * AT_BLK;  // 64 or 128
+    const int H = a.H, ld = 3 * H * AT_DK, ldo = H * AT_DK;
+    extern __shared__ __align__(16) __nv_bfloat16 at_smem[];
+    __nv_bfloat16 *qs = at_smem, *ks = qs + AF_ROWS * AT_PITCH, *vs = ks + AF_ROWS * AT_PITCH;
+    __nv_bfloat16 *dos = vs + AF_ROWS * AT_PITCH;
+    __nv_bfloat16 *ps = dos + AF_ROWS * AT_PITCH, *dss = ps + AF_ROWS * AT_PITCH;  // one 64-key block
+    float *dsh = reinterpret_cast<float *>(dss + AF_ROWS * AT_PITCH), *lse_s = dsh + AF_ROWS;
+    const __nv_bfloat16 *src = a.qkv + (long long)g * a.C * ld;
+    const long long ob = (long long)g * a.C * ldo;
+    // all 128 rows of each tile: rows past L are zero-filled (no global read)
+    at_cp_rows_n<AF_THREADS>(qs, src, ld, 0, AF_ROWS, L, h * AT_DK);
+    at_cp_rows_n<AF_THREADS>(dos, a.dout + ob, ldo, 0, AF_ROWS, L, h * AT_DK);
+    at_cp_rows_n<AF_THREADS>(ks, src, ld, 0, AF_ROWS, L, (H + h) * AT_DK);
+    at_cp_rows_n<AF_THREADS>(vs, src, ld, 0, AF_ROWS, L, (2 * H + h) * AT_DK);
+    at_cp_commit();
+    for (int i = threadIdx.x; i < AF_ROWS; i += AF_THREADS)
+        lse_s[i] = i < L ? __ldg(a.lse + ((long long)g * H + h) * a.C + i) : 0.0f;
+    // D = rowsum(dO * O): two threads per row, 32 columns each, in a fixed order
+    // (O straight from global memory; dO from shared memory once it has landed)
+    float oc[32];
+    {
+        const int r = threadIdx.x >> 1, c0 = (threadIdx.x & 1) * 32;
+#pragma unroll
+        for (int c = 0; c < 32; c += 8) {
+            uint4 v = make_uint4(0, 0, 0, 0);
+            if (r < L) v = __ldg(reinterpret_cast<const uint4 *>(a.o + ob + (long long)r * ldo + h * AT_DK + c0 + c));
+            bf16x8_to_f32(v, oc + c);
+        }
+    }
+    at_cp_wait(0);
+    {
+        const int r = threadIdx.x >> 1, c0 = (threadIdx.x & 1) * 32;
+        float acc = 0.0f;
+#pragma unroll 8
+        for (int c = 0; c < 32; ++c) acc += __bfloat162float(dos[r * AT_PITCH + c0 + c]) * oc[c];
+        acc += __shfl_xor_sync(0xffffffffu, acc, 1);
+        if ((threadIdx.x & 1) == 0) dsh[r] = acc;
+    }
+    __syncthreads();
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = lane & 3, g8 = lane >> 2;
+    const int row0 = warp * 16;
+    float lse[2], dd[2];
+    bool rv[2];
+#pragma unroll
+    for (int h2 = 0; h2 < 2; ++h2) {
+        const int r = row0 + g8 + 8 * h2;
+        rv[h2] = r < L;
+        lse[h2] = lse_s[r];
+        dd[h2] = dsh[r];
+    }
+    float dq[8][4];
+    at_zero(dq);
+    for (int kb = 0; kb < Lp; kb += AT_BLK) {
+        {
+            uint32_t fa[4][4];
+            float s[8][4], dp[8][4];
+            at_zero(s);
+            at_zero(dp);
+            at_afrag(fa, qs, row0);
+            at_mma_abt(s, fa, ks, kb);
+            at_afrag(fa, dos, row0);
+            at_mma_abt(dp, fa, vs, kb);
+#pragma unroll
+            for (int nt = 0; nt < 8; ++nt)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int key = kb + nt * 8 + 2 * t + (j & 1);
+                    const bool in = key < L && rv[j >> 1];
+                    const float p = in ? __expf(s[nt][j] * a.scale - lse[j >> 1]) : 0.0f;
+                    s[nt][j] = p;                                      // P
+                    dp[nt][j] = in ? p * (dp[nt][j] - dd[j >> 1]) : 0.0f;  // dS
+                }
+            at_mma_pb(dq, dp, ks, kb);
+            at_put(ps, row0, s);
+            at_put(dss, row0, dp);
+        }
+        __syncthreads();
+        {
+            float acc[8][4];
+            at_zero(acc);
+            const int key0 = (warp & 3) * 16;  // the warp's 16 keys of the block
+            if (warp < 4) {
+                at_mma_tb(acc, ps, key0, dos, Lp);   // dV = P^T dO
+                at_store(acc, 1.0f, a.dqkv + (long long)g * a.C * ld, ld, kb + key0, L, (2 * H + h) * AT_DK);
+            } else {
+                at_mma_tb(acc, dss, key0, qs, Lp);   // dK = dS^T Q / sqrt(dk)
+                at_store(acc, a.scale, a.dqkv + (long long)g * a.C * ld, ld, kb + key0, L, (H + h) * AT_DK);
+            }
+        }
+        __syncthreads();  // P and dS of this block are read; the next block rewrites them
+    }
+    at_store(dq, a.scale, a.dqkv + (long long)g * a.C * ld, ld, row0, L, h * AT_DK);
+}
+
 size_t at_smem_fwd(int C) {
     const int Cp = (C + AT_BLK - 1) / AT_BLK * AT_BLK;
     return (size_t)(AT_BLK + 2 * Cp) * AT_PITCH * 2;
@@ -410,6 +555,7 @@ size_t at_smem_dq(int C) {
     const int Cp = (C + AT_BLK - 1) / AT_BLK * AT_BLK;
     return (size_t)(3 * AT_BLK + 2 * Cp) * AT_PITCH * 2 + AT_BLK * 4;
 }
+size_t at_smem_fused() { return (size_t)6 * AF_ROWS * AT_PITCH * 2 + 2 * (size_t)AF_ROWS * 4; }
 size_t at_smem_dkv(int C) {
     const int Cp = (C + AT_BLK - 1) / AT_BLK * AT_BLK;
     return (size_t)(2 * AT_BLK + 2 * Cp) * AT_PITCH * 2 + 2 * (size_t)Cp * 4;
@@ -465,6 +611,19 @@ int launch_attn_core_bwd(int G, int C, int H, const int32_t *load, const __nv_bf
     a.dsum = dsum;
     a.dqkv = dqkv;
     a.scale = 1.0f / sqrtf((float)AT_DK);
+    if (C <= AF_ROWS) {  // every group fits one CTA: S, P, dP and dS formed once
+        static std::atomic<int> lim_f[64], carve_f[64];
+        const size_t smem = at_smem_fused();
+        if (const int st = raise_smem_limit((const void *)attn_bwd_fused_kernel, lim_f, (int)smem)) return st;
+        int dev = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64 && !carve_f[dev].exchange(1))
+            cudaFuncSetAttribute((const void *)attn_bwd_fused_kernel,
+                                 cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+        trace_before(s, "attn_bwd");
+        const int st = launch_kernel(attn_bwd_fused_kernel, dim3(1, H, G), dim3(AF_THREADS), smem, s, a);
+        trace_after(s);
+        return st;
+    }
     static std::atomic<int> lim_dq[64], lim_dkv[64], carve_dq[64], carve_dkv[64];
     int st = at_launch(attn_bwd_dq_kernel, a, at_smem_dq(C), lim_dq, carve_dq, s, "attn_bwd_dq");
     if (st != VMOE_OK) return st;
