@@ -488,7 +488,7 @@ def measure_attention(vm, cfg, heads, dev, stream, steps, warmup, peaks, seed):
     kst = {}
     for name, lst in per_kernel.items():
         kst[name] = {"launches": len(lst), "ms_avg": round(sum(lst) / len(lst), 5)}
-    core_ms = sum(kst[n]["ms_avg"] for n in ("attn_fwd", "attn_bwd_dq", "attn_bwd_dkv") if n in kst)
+    core_ms = sum(kst[n]["ms_avg"] for n in ("attn_fwd", "attn_bwd", "attn_bwd_dq", "attn_bwd_dkv") if n in kst)
     out = {"config": {"workload": cfg.name + " shape with attention experts (H=%d, head dim 64)" % heads,
                       "T": cfg.T, "tokens_per_task": cfg.N, "d_model": d, "E": cfg.E, "k": cfg.k,
                       "capacity": C, "heads": heads, "kept_assignments": A},
