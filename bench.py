@@ -743,11 +743,17 @@ def run_ours(args, cfg, rank, world, local_rank):
     if rank == 0 and world == 1 and not args.headline_only:
         del runner
         torch.cuda.empty_cache()
-        out["workloads"] = {name: measure_secondary(vm, workloads.CONFIGS[name], dev, stream,
-                                                    args.aux_steps, args.warmup, peaks, seed=7)
-                            for name in SECONDARY if name != cfg.name}
-        out["attention_experts"] = measure_attention(vm, workloads.CONFIGS[workloads.HEADLINE], 12, dev,
-                                                     stream, args.aux_steps, args.warmup, peaks, seed=9)
+        # a --tasks prefix (a profiling run) skips the other workloads and runs the
+        # attention experts on the same prefix of the headline workload
+        if not args.tasks:
+            out["workloads"] = {name: measure_secondary(vm, workloads.CONFIGS[name], dev, stream,
+                                                        args.aux_steps, args.warmup, peaks, seed=7)
+                                for name in SECONDARY if name != cfg.name}
+        att_cfg = workloads.CONFIGS[workloads.HEADLINE]
+        if args.tasks:
+            att_cfg = att_cfg.with_(T=min(args.tasks, att_cfg.T))
+        out["attention_experts"] = measure_attention(vm, att_cfg, 12, dev, stream, args.aux_steps,
+                                                     args.warmup, peaks, seed=9)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         out["cpu_baseline"] = cpu_baseline(cfg, budget_s=args.cpu_budget)
     if dist is not None:
