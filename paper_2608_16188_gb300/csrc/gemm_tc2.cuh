@@ -18,14 +18,18 @@
 // row tiles of the group; their A k-blocks stream through a ring.
 //
 // Roles, per CTA (320 threads):
-//   warp 0      TMA producer: its own A and B halves into its own shared memory,
-//               signalling its own `afull` / `bfull` barriers.
-//   warp 1      tail warp: waits for its copies, zeroes the K-tail rows past
-//               the group's load (padding rows may hold anything, NaN
-//               included), then arrives on the leader CTA's `aready` / `bready`
-//               (count 2: both CTAs).  In the leader (rank 0) lane 0 also issues
-//               the MMAs once both CTAs are ready and commits them with a
-//               multicast arrive on both CTAs' `aempty`, `bempty` and `tfull`.
+//   warp 0      TMA producer: its own A and B halves into its own shared memory.
+//               A k-blocks complete on the leader's `afull` (both CTAs' bytes).
+//               With two B buffers a B tile completes on this CTA's own `bfull`;
+//               with one (K > 128 rows) each k-block piece of a dense B tile
+//               completes on the leader's `bfull` of that piece, like A.
+//   warp 1      B hand-over: with two B buffers (and for compact B) it waits for
+//               this CTA's B copy, zeroes the rows of a compact B's first
+//               k-block that belong to a neighbour, then arrives on the leader's
+//               `bready` (count 2: both CTAs).  In the leader (rank 0) lane 0
+//               also issues the MMAs once both CTAs' operands are in and commits
+//               them with a multicast arrive on both CTAs' `aempty`, `bempty`
+//               (per piece with one B buffer) and `tfull`.
 //   warps 2-9   epilogue: tcgen05.ld of this CTA's 128 accumulator rows, arrive on
 //               the leader's `tempty` (count 16: 8 warps x 2 CTAs), bf16 packing
 //               and TMA bulk tensor stores from 128-byte-swizzled staging.
