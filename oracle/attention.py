@@ -73,17 +73,22 @@ def attention_expert_fwd(xe, wq, wk, wv, wo, load, heads):
     return out
 
 
-def attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, heads):
+def attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, heads, o=None):
     """Backward of every group: gradients of sum_g <dye[g], ye[g]> (valid rows).
 
     Returns dict dxe [G, C, d] (rows past the load zero), dwq, dwk, dwv [G, d, H*dk],
     dwo [G, H*dk, d] (zero for an empty group).  Chain rule, step by step:
         dO = dYe W_o^T,  dW_o = O^T dYe
         per head: dV_h = P_h^T dO_h,  dP_h = dO_h V_h^T,
-                  dS_h = P_h * (dP_h - rowsum(dP_h * P_h)),
+                  dS_h = P_h * (dP_h - D_h),  D_h = rowsum(dP_h * P_h),
                   dQ_h = dS_h K_h / sqrt(d_k),  dK_h = dS_h^T Q_h / sqrt(d_k)
         dXe = dQ W_q^T + dK W_k^T + dV W_v^T,
-        dW_q = Xe^T dQ,  dW_k = Xe^T dK,  dW_v = Xe^T dV."""
+        dW_q = Xe^T dQ,  dW_k = Xe^T dK,  dW_v = Xe^T dV.
+
+    o [G, C, H*dk], optional: the forward's O as stored by whoever ran the
+    forward, for a backward handed that O rather than recomputing it.  It then
+    stands in for O in dW_o and in D_h = rowsum(dO_h * O_h), which equals
+    rowsum(dP_h * P_h) when O_h = P_h V_h exactly (row i: sum_j P_ij dO_i.V_j)."""
     fw = attention_expert_fwd(xe, wq, wk, wv, wo, load, heads)
     xe, wq, wk, wv, wo, dye = map(_f64, (xe, wq, wk, wv, wo, dye))
     G, C, d = fw["ye"].shape
@@ -95,6 +100,7 @@ def attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, heads):
     dk = hd // heads
     ld = np.asarray(load).reshape(-1)
     scale = 1.0 / np.sqrt(dk)
+    o_given = None if o is None else _f64(o).reshape(G, C, hd)
     res = {"dxe": np.zeros((G, C, d)), "dwq": np.zeros((G, d, hd)), "dwk": np.zeros((G, d, hd)),
            "dwv": np.zeros((G, d, hd)), "dwo": np.zeros((G, hd, d))}
     for g in range(G):
@@ -102,16 +108,22 @@ def attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, heads):
         if L == 0:
             continue
         x, dy = xe[g, :L], dye[g, :L]
-        q, k, v, o = (fw[n][g, :L] for n in ("q", "k", "v", "o"))
+        q, k, v, og = (fw[n][g, :L] for n in ("q", "k", "v", "o"))
+        if o_given is not None:
+            og = o_given[g, :L]
         do = dy @ wo[g].T
-        res["dwo"][g] = o.T @ dy
+        res["dwo"][g] = og.T @ dy
         dq, dkk, dv = np.zeros((L, hd)), np.zeros((L, hd)), np.zeros((L, hd))
         for h in range(heads):
             c = slice(h * dk, (h + 1) * dk)
             p = fw["p"][g, h, :L, :L]
             dv[:, c] = p.T @ do[:, c]
             dp = do[:, c] @ v[:, c].T
-            ds = p * (dp - (dp * p).sum(axis=1, keepdims=True))
+            if o_given is None:
+                dd = (dp * p).sum(axis=1, keepdims=True)
+            else:
+                dd = (do[:, c] * og[:, c]).sum(axis=1, keepdims=True)
+            ds = p * (dp - dd)
             dq[:, c] = (ds @ k[:, c]) * scale
             dkk[:, c] = (ds.T @ q[:, c]) * scale
         res["dxe"][g, :L] = dq @ wq[g].T + dkk @ wk[g].T + dv @ wv[g].T

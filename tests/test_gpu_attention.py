@@ -7,13 +7,16 @@ Every stage is compared with the oracle given the inputs that stage received on
 the GPU: the Q/K/V projection, the attention core (O from the GPU's Q, K, V -- the
 oracle is handed [Q | K | V] as its token block with 0/1 selector weights, so its
 projections reproduce them exactly), the output projection, and in the backward
-dO, the core's dQ, dK, dV (from the GPU's Q, K, V and dO), dXe, dW_qkv and dW_o.
+dO, the core's dQ, dK, dV (from the GPU's Q, K, V, dO and the stored O the
+backward call received, which enters through D = rowsum(dO * O)), dXe, dW_qkv and
+dW_o.
 Ye is also compared end to end with the oracle run from Xe and the weights alone.
 Cases: a capacity of 188 rows (three ragged 64-row blocks in the core, two row
 tiles in the GEMMs) and of 500 rows (eight key blocks; Zipf-skewed loads), which
 take the two-kernel backward; capacities of 125 rows (one or two key blocks a
 group) and of 12 rows with 16 of 32 groups empty (Zipf-skewed), which take the fused
-backward of groups of at most 128 tokens.
+backward of groups of at most 128 tokens; and the benchmark's per-group shape (d 768,
+12 heads, capacity 124).
 """
 import numpy as np
 import pytest
@@ -36,6 +39,9 @@ CASES = {
                          bias="drift"), 2),
     "attn_c12_empty": (Config("attn_c12", 63, T=2, N=96, d=128, f=128, E=16, k=1, cf=2.0, dtype="bf16",
                               bias="zipf"), 2),
+    # the benchmark's per-group shape: ViT-B (d 768), 12 heads, C 124
+    "attn_vitb_h12": (Config("attn_vitb", 64, T=2, N=394, d=768, f=128, E=8, k=2, cf=1.25, dtype="bf16",
+                             bias="drift"), 12),
 }
 DK = 64
 
@@ -54,10 +60,11 @@ def _weights(cfg, H, seed):
     return wqkv, wo
 
 
-def _core_oracle(qkv, load, H, dout=None):
+def _core_oracle(qkv, load, H, dout=None, o=None):
     """The oracle's attention core on the given Q|K|V rows: [Q|K|V] as the token
     block, weights selecting each third and W_o = [I 0 0], so its q, k, v are the
-    given ones exactly and its Ye starts with O."""
+    given ones exactly and its Ye starts with O.  The backward takes the O it is
+    given (the one the GPU's backward was handed) for D = rowsum(dO * O)."""
     G, C, w3 = qkv.shape
     hd = w3 // 3
     eye = np.eye(hd)
@@ -71,7 +78,7 @@ def _core_oracle(qkv, load, H, dout=None):
         return fw["ye"][..., :hd], None
     dye = np.zeros((G, C, w3))
     dye[..., :hd] = dout  # so that dO = dYe W_o^T = dout
-    bw = att.attention_expert_bwd(qkv, wq, wk, wv, wo, dye, load, H)
+    bw = att.attention_expert_bwd(qkv, wq, wk, wv, wo, dye, load, H, o=o)
     return fw["ye"][..., :hd], bw["dxe"]  # O, and [dQ | dK | dV]
 
 
@@ -117,7 +124,7 @@ def test_attention_experts_stagewise(name):
     ref_dout = np.einsum("gcd,ghd->gch", dye64, wo64)
     dout64 = np64(ws[:G * C * hd * 2].view(torch.bfloat16)).reshape(G, C, hd)
     dout64[~rows] = 0.0
-    _, ref_dqkv = _core_oracle(qkv64, load, H, dout64)
+    _, ref_dqkv = _core_oracle(qkv64, load, H, dout64, o64)
     dqkv64 = np64(ws[G * C * hd * 2:G * C * hd * 2 + G * C * 3 * hd * 2].view(torch.bfloat16)).reshape(G, C, 3 * hd)
     dqkv64[~rows] = 0.0
     ref_dxe = np.einsum("gce,gde->gcd", dqkv64, wqkv64)

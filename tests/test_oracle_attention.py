@@ -121,3 +121,53 @@ def test_permutation_equivariance_padding_and_empty_groups():
     xj = xe.copy()
     xj[1, 5:] = -7.0
     assert np.array_equal(att.attention_expert_fwd(xj, wq, wk, wv, wo, load, H)["ye"], fw["ye"])
+
+
+def test_stored_o_enters_only_through_d_and_dwo():
+    """The backward handed the forward's O: the exact O reproduces the default
+    (rowsum(dO_h * O_h) = rowsum(dP_h * P_h) when O_h = P_h V_h); an O moved
+    orthogonally to dO in every head row leaves D, hence dXe and dW_q,k,v, as
+    they were and moves dW_o by (the move)^T dYe; a move along dO shifts each
+    row's dS by -P_ij r_i, with r_i the change of D_i."""
+    xe, wq, wk, wv, wo, dye, load, H = _case(6)
+    fw = att.attention_expert_fwd(xe, wq, wk, wv, wo, load, H)
+    base = att.attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, H)
+    same = att.attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, H, o=fw["o"])
+    for n in base:
+        np.testing.assert_allclose(same[n], base[n], rtol=1e-10, atol=1e-12)
+    G, C, d = xe.shape
+    hd = wq.shape[-1]
+    dk = hd // H
+    rng = np.random.default_rng(11)
+    do = np.einsum("gcd,ghd->gch", dye, wo)
+    delta = np.zeros((G, C, hd))
+    for g in range(G):
+        L = int(load[g])
+        for h in range(H):
+            c = slice(h * dk, (h + 1) * dk)
+            r = rng.standard_normal((L, dk))
+            u = do[g, :L, c]
+            delta[g, :L, c] = r - (r * u).sum(1, keepdims=True) / (u * u).sum(1, keepdims=True) * u
+    orth = att.attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, H, o=fw["o"] + delta)
+    for n in ("dxe", "dwq", "dwk", "dwv"):
+        np.testing.assert_allclose(orth[n], base[n], rtol=1e-10, atol=1e-12)
+    rows = (np.arange(C)[None, :] < load[:, None])[..., None]
+    np.testing.assert_allclose(orth["dwo"] - base["dwo"], np.einsum("gch,gcd->ghd", delta, dye * rows),
+                               rtol=1e-10, atol=1e-12)
+    # along dO: D_i of head h grows by r_i = 0.1 |dO_i,h|^2, so dQ_h moves by -diag(r) P_h K_h / sqrt(d_k)
+    along = att.attention_expert_bwd(xe, wq, wk, wv, wo, dye, load, H, o=fw["o"] + 0.1 * do * rows)
+    np.testing.assert_allclose(along["dwv"], base["dwv"], rtol=1e-10, atol=1e-12)
+    want = base["dwq"].copy()
+    for g in range(G):
+        L = int(load[g])
+        if L == 0:
+            continue
+        x = xe[g, :L]
+        q, k = x @ wq[g], x @ wk[g]
+        dq = np.zeros((L, hd))
+        for h in range(H):
+            c = slice(h * dk, (h + 1) * dk)
+            r = 0.1 * (do[g, :L, c] ** 2).sum(1, keepdims=True)
+            dq[:, c] = -(r * fw["p"][g, h, :L, :L]) @ k[:, c] / np.sqrt(dk)
+        want[g] += x.T @ dq
+    np.testing.assert_allclose(along["dwq"], want, rtol=1e-9, atol=1e-11)
