@@ -15,8 +15,9 @@ Cases: a capacity of 188 rows (three ragged 64-row blocks in the core, two row
 tiles in the GEMMs) and of 500 rows (eight key blocks; Zipf-skewed loads), which
 take the two-kernel backward; capacities of 125 rows (one or two key blocks a
 group) and of 12 rows with 16 of 32 groups empty (Zipf-skewed), which take the fused
-backward of groups of at most 128 tokens; and the benchmark's per-group shape (d 768,
-12 heads, capacity 124).
+backward of groups of at most 128 tokens; the benchmark's per-group shape (d 768,
+12 heads, capacity 124); and dY scaled by 2^-24 and by 2^12 (exact powers of two),
+which the backward's fp16 operands meet only through their per-CTA scales.
 """
 import numpy as np
 import pytest
@@ -42,6 +43,12 @@ CASES = {
     # the benchmark's per-group shape: ViT-B (d 768), 12 heads, C 124
     "attn_vitb_h12": (Config("attn_vitb", 64, T=2, N=394, d=768, f=128, E=8, k=2, cf=1.25, dtype="bf16",
                              bias="drift"), 12),
+    # dY times 2^-24 (dO near 1e-8): below fp16's normal range unless the backward
+    # scales its operands; and dY times 2^12 (dO near 1e4, dS beyond fp16's range)
+    "attn_c125_tiny_dy": (Config("attn_c125t", 65, T=2, N=400, d=256, f=128, E=8, k=2, cf=1.25, dtype="bf16",
+                                 bias="drift"), 4, 2.0 ** -24),
+    "attn_c188_huge_dy": (Config("attn_c188h", 66, T=2, N=300, d=256, f=128, E=4, k=2, cf=1.25, dtype="bf16",
+                                 bias="drift"), 2, 2.0 ** 12),
 }
 DK = 64
 
@@ -85,11 +92,13 @@ def _core_oracle(qkv, load, H, dout=None, o=None):
 @pytest.mark.parametrize("name", list(CASES))
 def test_attention_experts_stagewise(name):
     import paper_2608_16188_gb300 as vm
-    cfg, H = CASES[name]
+    cfg, H = CASES[name][:2]
+    dy_scale = CASES[name][2] if len(CASES[name]) > 2 else 1.0
     hd = H * DK
     p = problem_of(cfg)
     C = vm.vmoe_problem_capacity(p)
     inp = to_dev(workloads.make_inputs(cfg, with_weights=False))
+    inp["dy"] = inp["dy"] * dy_scale  # a power of two: exact in bf16
     wqkv, wo = _weights(cfg, H, 7)
     wqkv_d, wo_d = wqkv.cuda(), wo.cuda()
     T, E, d, G = cfg.T, cfg.E, cfg.d, cfg.T * cfg.E
