@@ -248,7 +248,10 @@ size_t vmoe_attn_expert_bwd_workspace_size(const vmoe_problem *p, int heads);
  *   dO = dYe W_o^T,  dW_o = O^T dYe,  D = rowsum(dO * O) per head,
  *   dS = P * (dO_h V_h^T - D),  dQ_h = dS K_h / 8,  dK_h = dS^T Q_h / 8,  dV_h = P^T dO_h,
  *   dXe = dQKV W_qkv^T,  dW_qkv = Xe^T dQKV,
- * P rebuilt from qkv and lse.  Inputs as written by the forward (xe, qkv, o, lse)
+ * P rebuilt from qkv and lse, D formed from the stored o.  The attention core's
+ * products take fp16 operands, each staged tile of Q, K, V and dO scaled by a
+ * power of two (exact for bf16 values), so P and dS enter dV, dQ and dK with 11
+ * significant bits; sums accumulate in fp32.  Inputs as written by the forward (xe, qkv, o, lse)
  * and dye [T,E,C,d] (vmoe_dispatch of dY with the gates); outputs dxe [T,E,C,d]
  * (rows >= load not written), dwqkv [T,E,d,3H64] and dwo [T,E,H64,d] (zero for an
  * empty group).  workspace: caller-owned device scratch of at least
