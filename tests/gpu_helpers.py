@@ -80,7 +80,8 @@ def rms_err(gpu, ref, mask=None, groups=None):
 
 def literal_err(gpu, ref, mask=None, groups=None):
     """max_i |gpu_i - ref_i| / rms(ref) over the whole tensor (the selected rows):
-    the tolerance of the benchmark spec read literally, one RMS per output tensor.
+    the 2e-2 tolerance ("normalised by each output's RMS") read literally, one
+    RMS per output tensor.
     Reported beside rel_err by the parity tests; the bar is rel_err's."""
     g, r, m = _pair(gpu, ref, mask, None if mask is None else groups)
     if m is not None:
