@@ -251,8 +251,10 @@ size_t vmoe_attn_expert_bwd_workspace_size(const vmoe_problem *p, int heads);
  * P rebuilt from qkv and lse, D formed from the stored o.  The attention core's
  * products take fp16 operands, each staged tile of Q, K, V and dO scaled by a
  * power of two (exact for bf16 values), so P and dS enter dV, dQ and dK with 11
- * significant bits; sums accumulate in fp32.  Inputs as written by the forward (xe, qkv, o, lse)
- * and dye [T,E,C,d] (vmoe_dispatch of dY with the gates); outputs dxe [T,E,C,d]
+ * significant bits; for C > 128, dQ = dS K instead takes dS as a bf16 value
+ * plus its bf16 residual.  Sums accumulate in fp32.  Inputs as written by the
+ * forward (xe, qkv, o, lse) and dye [T,E,C,d] (vmoe_dispatch of dY with the
+ * gates); outputs dxe [T,E,C,d]
  * (rows >= load not written), dwqkv [T,E,d,3H64] and dwo [T,E,H64,d] (zero for an
  * empty group).  workspace: caller-owned device scratch of at least
  * vmoe_attn_expert_bwd_workspace_size(p, heads) bytes (else VMOE_ERR_INVALID),

@@ -14,14 +14,21 @@
 // The projections and their gradients are the grouped tcgen05 GEMMs of the FFN
 // experts (row mode and weight-gradient mode).  The attention core is here:
 // flash-attention style kernels on mma.sync (m16n8k16, fp32 accumulate; bf16
-// operands in the forward, power-of-two-scaled fp16 in the backward), one CTA
-// per (group, head, block of 64 rows), 4 warps of 16 rows.  Each CTA keeps the whole group's keys (or queries) of its head in
+// operands in the forward, power-of-two-scaled fp16 in most of the backward),
+// one CTA per (group, head, block of 64 rows), 4 warps of 16 rows.  Each CTA
+// keeps the whole group's keys (or queries) of its head in
 // shared memory -- a group holds at most C <= 512 tokens -- so the softmax of a
 // row runs online over key blocks of 64 with the row maximum subtracted, and
 // the forward saves each row's log-sum-exp for the backward to rebuild P.
-// The tiles arrive by cp.async; in the forward, one commit group per block of
-// 64 keys, so the work on block j overlaps the copies of the blocks after it
-// (the backward waits for all of them: its operand scales span every row).
+// The tiles arrive by cp.async; in the forward and the dQ kernel, one commit
+// group per block of 64 keys, so the work on block j overlaps the copies of the
+// blocks after it (dK/dV and the fused backward wait for all of theirs: their
+// operand scales span every row).  The dQ kernel of groups above 128 tokens
+// keeps bf16 operands and takes dS as a bf16 value plus its bf16 residual, two
+// products.  In fp16, every query block's CTA would scale the whole of K and V
+// (measured at 8 tasks and C 248: 245 us with the residual, against 297 us
+// with K and V scaled once all keys have landed, 326 us with each key block
+// scaled as it lands, and 206 us for bf16 with a single product).
 // Keys (or queries) past the load are masked; rows past it are never stored.
 // There are no atomics: dQ is one kernel over query blocks, dK and dV another
 // over key blocks, so every sum runs in a fixed order.
@@ -300,8 +307,8 @@ __global__ void __launch_bounds__(AT_THREADS) attn_fwd_kernel(AtArgs a) {
 }
 
 // ------------------------------------------------------------------ backward operands
-// The backward's products take fp16 operands, each staged tile scaled by its own
-// power of two.  The inputs are bf16 (8 significant bits), so a bf16 value
+// The fused backward and the dK/dV kernel take fp16 operands, each staged tile
+// scaled by its own power of two (the dQ kernel keeps bf16, see the header).  The inputs are bf16 (8 significant bits), so a bf16 value
 // times 2^e converts to fp16 (11 bits) exactly while it stays an fp16 normal;
 // the products, exact in either type, are then those of the bf16 path.  What
 // changes is the two values the kernels round for the second products, P (for
@@ -417,9 +424,20 @@ __device__ __forceinline__ AtScales at_scales(const uint32_t (&m)[5], float scal
     return sc;
 }
 
+// v - bf16(v), in place: the part of a value its bf16 rounding drops (dS as
+// value + residual carries about 16 significant bits into dQ = dS K).
+template <int NT>
+__device__ __forceinline__ void at_residual(float (&v)[NT][4]) {
+#pragma unroll
+    for (int i = 0; i < NT; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) v[i][j] -= __bfloat162float(__float2bfloat16_rn(v[i][j]));
+}
+
 // ------------------------------------------------------------------ backward: dQ (and D)
 // CTA (query block, head, group): D = rowsum(dO * O) of its 64 queries, then
-// dQ = sum over key blocks of dS K, dS = P * (dO V^T - D), P = exp(S - lse).
+// dQ = sum over key blocks of dS K, dS = P * (dO V^T - D), P = exp(S - lse);
+// bf16 operands, dS entering dQ as a bf16 value and its residual.
 __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kernel(AtArgs a) {
     pdl_wait();
     const int qb = blockIdx.x, h = blockIdx.y, g = blockIdx.z;
@@ -432,7 +450,6 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
     __nv_bfloat16 *qs = at_smem, *dos = qs + AT_BLK * AT_PITCH, *os = dos + AT_BLK * AT_PITCH;
     __nv_bfloat16 *ks = os + AT_BLK * AT_PITCH, *vs = ks + Lp * AT_PITCH;
     float *dsh = reinterpret_cast<float *>(vs + Lp * AT_PITCH);  // [64] D of the block
-    uint32_t *red = reinterpret_cast<uint32_t *>(dsh + AT_BLK);   // [5][4] block maxima
     const __nv_bfloat16 *src = a.qkv + (long long)g * a.C * ld;
     const long long ob = (long long)g * a.C * ldo;
     // commit group 0: this block's Q, dO, O and key block 0; group j: key block j
@@ -445,9 +462,8 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
         at_cp_rows(vs + j * AT_BLK * AT_PITCH, src, ld, j * AT_BLK, AT_BLK, L, (2 * H + h) * AT_DK);
         at_cp_commit();
     }
-    at_cp_wait(0);  // every key: the scales of K and V span them all
+    at_cp_wait(nkb - 1);
     // D: two threads per row, 32 columns each, in a fixed order
-    float dabs;
     {
         const int r = threadIdx.x >> 1, c0 = (threadIdx.x & 1) * 32;
         float acc = 0.0f;
@@ -455,22 +471,11 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
         for (int c = 0; c < 32; ++c)
             acc += __bfloat162float(dos[r * AT_PITCH + c0 + c]) * __bfloat162float(os[r * AT_PITCH + c0 + c]);
         acc += __shfl_xor_sync(0xffffffffu, acc, 1);
-        dabs = fabsf(acc);
         if ((threadIdx.x & 1) == 0) {
             dsh[r] = acc;
             if (q0 + r < L) a.dsum[((long long)g * H + h) * a.C + q0 + r] = acc;
         }
     }
-    // the operands as scaled fp16 (D is formed from the bf16 dO first)
-    uint32_t mx[5] = {at_tile_absmax<AT_THREADS>(qs, AT_BLK), at_tile_absmax<AT_THREADS>(ks, Lp),
-                      at_tile_absmax<AT_THREADS>(vs, Lp), at_tile_absmax<AT_THREADS>(dos, AT_BLK),
-                      __float_as_uint(dabs)};
-    at_block_max<5, AT_THREADS / 32>(mx, red);
-    const AtScales sc = at_scales(mx, a.scale);
-    at_tile_to_f16<AT_THREADS>(qs, AT_BLK, sc.q);
-    at_tile_to_f16<AT_THREADS>(ks, Lp, sc.k);
-    at_tile_to_f16<AT_THREADS>(vs, Lp, sc.v);
-    at_tile_to_f16<AT_THREADS>(dos, AT_BLK, sc.dO);
     __syncthreads();
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, t = lane & 3, g8 = lane >> 2;
     uint32_t qa[4][4], da[4][4];
@@ -481,27 +486,30 @@ __global__ void __launch_bounds__(AT_THREADS, AT_MIN_CTAS_BWD) attn_bwd_dq_kerne
     for (int h2 = 0; h2 < 2; ++h2) {
         const int rl = warp * 16 + g8 + 8 * h2, r = q0 + rl;
         lse[h2] = r < L ? __ldg(a.lse + ((long long)g * H + h) * a.C + r) : 0.0f;
-        dd[h2] = dsh[rl] * sc.d;
+        dd[h2] = dsh[rl];
     }
     float dq[8][4];
     at_zero(dq);
     for (int kb = 0; kb < Lp; kb += AT_BLK) {
+        if (kb > 0) at_cp_wait(nkb - 1 - kb / AT_BLK);
         float s[8][4], dp[8][4];
         at_zero(s);
         at_zero(dp);
-        at_mma_abt<true>(s, qa, ks, kb);
-        at_mma_abt<true>(dp, da, vs, kb);
+        at_mma_abt<false>(s, qa, ks, kb);
+        at_mma_abt<false>(dp, da, vs, kb);
 #pragma unroll
         for (int nt = 0; nt < 8; ++nt)
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int key = kb + nt * 8 + 2 * t + (j & 1);
-                const float p = key < L ? __expf(s[nt][j] * sc.s - lse[j >> 1]) : 0.0f;
-                s[nt][j] = p * (dp[nt][j] * sc.dp - dd[j >> 1]);  // dS, scaled
+                const float p = key < L ? __expf(s[nt][j] * a.scale - lse[j >> 1]) : 0.0f;
+                s[nt][j] = p * (dp[nt][j] - dd[j >> 1]);  // dS
             }
-        at_mma_pb<true>(dq, s, ks, kb);
+        at_mma_pb<false>(dq, s, ks, kb);  // dS as bf16 value
+        at_residual(s);
+        at_mma_pb<false>(dq, s, ks, kb);  // and its residual
     }
-    at_store(dq, sc.dq, a.dqkv + (long long)g * a.C * ld, ld, q0 + warp * 16, L, h * AT_DK);
+    at_store(dq, a.scale, a.dqkv + (long long)g * a.C * ld, ld, q0 + warp * 16, L, h * AT_DK);
 }
 
 // ------------------------------------------------------------------ backward: dK, dV
@@ -733,7 +741,7 @@ size_t at_smem_fwd(int C) {
 }
 size_t at_smem_dq(int C) {
     const int Cp = (C + AT_BLK - 1) / AT_BLK * AT_BLK;
-    return (size_t)(3 * AT_BLK + 2 * Cp) * AT_PITCH * 2 + AT_BLK * 4 + 5 * (AT_THREADS / 32) * 4;
+    return (size_t)(3 * AT_BLK + 2 * Cp) * AT_PITCH * 2 + AT_BLK * 4;
 }
 size_t at_smem_fused() {
     return (size_t)6 * AF_ROWS * AT_PITCH * 2 + 2 * (size_t)AF_ROWS * 4 + 5 * (AF_THREADS / 32) * 4;
