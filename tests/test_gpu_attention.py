@@ -17,7 +17,9 @@ take the two-kernel backward; capacities of 125 rows (one or two key blocks a
 group) and of 12 rows with 16 of 32 groups empty (Zipf-skewed), which take the fused
 backward of groups of at most 128 tokens; the benchmark's per-group shape (d 768,
 12 heads, capacity 124); and dY scaled by 2^-24 and by 2^12 (exact powers of two),
-which the backward's fp16 operands meet only through their per-CTA scales.
+which the backward's fp16 operands meet only through their per-CTA scales.  At full
+size, the benchmark's attention leg (17 tasks, 544 groups) is checked on sampled
+groups the oracle recomputes one by one.
 """
 import numpy as np
 import pytest
@@ -89,6 +91,74 @@ def _core_oracle(qkv, load, H, dout=None, o=None):
     return fw["ye"][..., :hd], bw["dxe"]  # O, and [dQ | dK | dV]
 
 
+def _host(groups, G, C, d, H, b, qkv, o, ye, lse, ws, dxe, dwqkv, dwo, wqkv, wo):
+    """fp64 host copies of the given groups' slices of every tensor of one
+    attention-expert step (dO and dQKV from the backward's workspace)."""
+    hd = H * DK
+    idx = torch.as_tensor(np.asarray(groups), dtype=torch.long)
+
+    def pick(t, *shape):
+        t = t.reshape(G, *shape)
+        return np64(t[idx.to(t.device)])
+    return {"xe": pick(b.xe, C, d), "dye": pick(b.dye, C, d), "qkv": pick(qkv, C, 3 * hd),
+            "o": pick(o, C, hd), "ye": pick(ye, C, d), "lse": pick(lse, H, C),
+            "dout": pick(ws[:G * C * hd * 2].view(torch.bfloat16), C, hd),
+            "dqkv": pick(ws[G * C * hd * 2:G * C * hd * 8].view(torch.bfloat16), C, 3 * hd),
+            "dxe": pick(dxe, C, d), "dwqkv": pick(dwqkv, d, 3 * hd), "dwo": pick(dwo, hd, d),
+            "wqkv": pick(wqkv, d, 3 * hd), "wo": pick(wo, hd, d)}
+
+def _compare_stages(name, H, load, rows, h):
+    """Every stage of the attention experts on the groups given (host fp64 copies
+    of the GPU's tensors in h, group-major), each against the oracle fed the
+    inputs that GPU stage received; then each valid row's log-sum-exp."""
+    G, C, d = h["xe"].shape
+    hd = H * DK
+    xe64, dye64, wqkv64, wo64 = h["xe"], h["dye"], h["wqkv"].reshape(G, d, 3 * hd), h["wo"].reshape(G, hd, d)
+    qkv64, o64, dout64, dqkv64 = h["qkv"].copy(), h["o"].copy(), h["dout"].copy(), h["dqkv"].copy()
+    for a in (qkv64, o64, dout64, dqkv64):
+        a[~rows] = 0.0
+    # stage by stage, each from the inputs that GPU stage received
+    ref_qkv = np.einsum("gcd,gde->gce", xe64, wqkv64)
+    ref_o, _ = _core_oracle(qkv64, load, H)
+    ref_ye = np.einsum("gch,ghd->gcd", o64, wo64)
+    ref_dout = np.einsum("gcd,ghd->gch", dye64, wo64)
+    _, ref_dqkv = _core_oracle(qkv64, load, H, dout64, o64)
+    ref_dxe = np.einsum("gce,gde->gcd", dqkv64, wqkv64)
+    ref_dwqkv = np.einsum("gcd,gce->gde", xe64 * rows[..., None], dqkv64)
+    ref_dwo = np.einsum("gch,gcd->ghd", o64, dye64 * rows[..., None])
+    # end to end from Xe and the weights
+    e2e = att.attention_expert_fwd(xe64, wqkv64[..., :hd], wqkv64[..., hd:2 * hd], wqkv64[..., 2 * hd:],
+                                   wo64, load, H)
+    checks = {
+        "qkv": (h["qkv"], ref_qkv, rows), "o": (h["o"], ref_o, rows), "ye": (h["ye"], ref_ye, rows),
+        "dout": (dout64, ref_dout, rows), "dqkv": (dqkv64, ref_dqkv, rows),
+        "dxe": (h["dxe"], ref_dxe, rows), "dwqkv": (h["dwqkv"], ref_dwqkv, None),
+        "dwo": (h["dwo"], ref_dwo, None), "ye_e2e": (h["ye"], e2e["ye"], rows),
+    }
+    # Every stage is held to the per-element bar; Ye end to end compounds three bf16
+    # roundings the interface fixes (QKV and O stored in bf16, P rounded for P V) and
+    # is held to the aggregate bar, its per-element figure reported.
+    bad = {}
+    for k_, (gpu, ref, m) in checks.items():
+        rel, rms = report(name, k_, np.asarray(gpu).reshape(G, -1), ref.reshape(G, -1), m, G)
+        if not ((rel <= BF16_TOL or k_ == "ye_e2e") and rms <= BF16_RMS_TOL):
+            bad[k_] = (rel, rms)
+    assert not bad, bad
+    # log-sum-exp of every valid row against the oracle's scores
+    lse64 = h["lse"].reshape(G, H, C)
+    for g in range(G):
+        L = int(load[g])
+        if L == 0:
+            continue  # an empty group has no rows
+        for hh in range(H):
+            q = qkv64[g, :L, hh * DK:(hh + 1) * DK]
+            k = qkv64[g, :L, hd + hh * DK:hd + (hh + 1) * DK]
+            s = q @ k.T / np.sqrt(DK)
+            m = s.max(axis=1)
+            ref = m + np.log(np.exp(s - m[:, None]).sum(axis=1))
+            np.testing.assert_allclose(lse64[g, hh, :L], ref, rtol=0, atol=2e-5)
+
+
 @pytest.mark.parametrize("name", list(CASES))
 def test_attention_experts_stagewise(name):
     import paper_2608_16188_gb300 as vm
@@ -121,57 +191,8 @@ def test_attention_experts_stagewise(name):
     else:  # groups of one and of two 64-key blocks, or empty groups, in the fused backward
         assert load.min() <= 64 and (load.max() > 64 or (load == 0).any()), load
     rows = valid_rows(load.reshape(T, E), C).reshape(G, C)
-    xe64, dye64 = np64(b.xe).reshape(G, C, d), np64(b.dye).reshape(G, C, d)
-    wqkv64, wo64 = np64(wqkv).reshape(G, d, 3 * hd), np64(wo).reshape(G, hd, d)
-    qkv64, o64 = np64(qkv).reshape(G, C, 3 * hd), np64(o).reshape(G, C, hd)
-    qkv64[~rows] = 0.0
-    o64[~rows] = 0.0
-    # stage by stage, each from the inputs that GPU stage received
-    ref_qkv = np.einsum("gcd,gde->gce", xe64, wqkv64)
-    ref_o, _ = _core_oracle(qkv64, load, H)
-    ref_ye = np.einsum("gch,ghd->gcd", o64, wo64)
-    ref_dout = np.einsum("gcd,ghd->gch", dye64, wo64)
-    dout64 = np64(ws[:G * C * hd * 2].view(torch.bfloat16)).reshape(G, C, hd)
-    dout64[~rows] = 0.0
-    _, ref_dqkv = _core_oracle(qkv64, load, H, dout64, o64)
-    dqkv64 = np64(ws[G * C * hd * 2:G * C * hd * 2 + G * C * 3 * hd * 2].view(torch.bfloat16)).reshape(G, C, 3 * hd)
-    dqkv64[~rows] = 0.0
-    ref_dxe = np.einsum("gce,gde->gcd", dqkv64, wqkv64)
-    ref_dwqkv = np.einsum("gcd,gce->gde", xe64 * rows[..., None], dqkv64)
-    ref_dwo = np.einsum("gch,gcd->ghd", o64, dye64 * rows[..., None])
-    # end to end from Xe and the weights
-    e2e = att.attention_expert_fwd(xe64, wqkv64[..., :hd], wqkv64[..., hd:2 * hd], wqkv64[..., 2 * hd:],
-                                   wo64, load, H)
-    checks = {
-        "qkv": (qkv, ref_qkv, rows), "o": (o, ref_o, rows), "ye": (ye, ref_ye, rows),
-        "dout": (dout64, ref_dout, rows), "dqkv": (dqkv64, ref_dqkv, rows),
-        "dxe": (dxe, ref_dxe, rows), "dwqkv": (dwqkv, ref_dwqkv, None), "dwo": (dwo, ref_dwo, None),
-        "ye_e2e": (ye, e2e["ye"], rows),
-    }
-    # Every stage is held to the per-element bar; Ye end to end compounds three bf16
-    # roundings the interface fixes (QKV and O stored in bf16, P rounded for P V) and
-    # is held to the aggregate bar, its per-element figure reported.
-    bad = {}
-    for k_, (gpu, ref, m) in checks.items():
-        g_ = np64(gpu) if isinstance(gpu, torch.Tensor) else gpu
-        rel, rms = report(name, k_, g_.reshape(G, -1), ref.reshape(G, -1),
-                          None if m is None else m, G)
-        if not ((rel <= BF16_TOL or k_ == "ye_e2e") and rms <= BF16_RMS_TOL):
-            bad[k_] = (rel, rms)
-    assert not bad, bad
-    # log-sum-exp of every valid row against the oracle's scores
-    lse64 = np64(lse).reshape(G, H, C)
-    for g in range(G):
-        L = int(load[g])
-        if L == 0:
-            continue  # an empty group has no rows
-        for h in range(H):
-            q = qkv64[g, :L, h * DK:(h + 1) * DK]
-            k = qkv64[g, :L, hd + h * DK:hd + (h + 1) * DK]
-            s = q @ k.T / np.sqrt(DK)
-            m = s.max(axis=1)
-            ref = m + np.log(np.exp(s - m[:, None]).sum(axis=1))
-            np.testing.assert_allclose(lse64[g, h, :L], ref, rtol=0, atol=2e-5)
+    _compare_stages(name, H, load, rows, _host(np.arange(G), G, C, d, H, b, qkv, o, ye, lse, ws, dxe, dwqkv, dwo,
+                                               wqkv, wo))
     # empty groups (where the routing left some): zero weight gradients; padding
     # rows of the outputs untouched
     empty = torch.from_numpy(load == 0)
@@ -180,3 +201,40 @@ def test_attention_experts_stagewise(name):
     pad = torch.from_numpy(~rows)
     assert torch.all(torch.isnan(ye.view(G, C, d).cpu()[pad]))
     assert torch.all(torch.isnan(dxe.view(G, C, d).cpu()[pad]))
+
+
+def test_attention_fullsize_sampled():
+    """The attention-expert leg the benchmark times -- the 17-task ViT-B shape with
+    12 heads of 64, C 124, the weights drawn on the device as there -- checked stage
+    by stage on sampled groups (the first, a middle and the last, the fullest and
+    the emptiest) that the oracle recomputes one by one."""
+    import paper_2608_16188_gb300 as vm
+    cfg = workloads.CONFIGS["vitb_t17"]
+    H = 12
+    hd = H * DK
+    p = problem_of(cfg)
+    C = vm.vmoe_problem_capacity(p)
+    inp = to_dev(workloads.make_inputs(cfg.with_(capacity=C), with_weights=False))
+    T, E, d, G = cfg.T, cfg.E, cfg.d, cfg.T * cfg.E
+    gen = torch.Generator(device="cuda")
+    gen.manual_seed(11)
+    wqkv = (torch.randn((G, d, 3 * hd), generator=gen, device="cuda") / d ** 0.5).to(torch.bfloat16)
+    wo = (torch.randn((G, hd, d), generator=gen, device="cuda") / hd ** 0.5).to(torch.bfloat16)
+    b = vm.Buffers(p)
+    vm.vmoe_route(p, inp["x"], inp["w_router"], inp["bias"], b.logits, b.idx, b.gate, b.slot, b.load)
+    vm.vmoe_dispatch(p, inp["x"], None, b.idx, b.slot, b.load, b.xe)
+    vm.vmoe_dispatch(p, inp["dy"], b.gate, b.idx, b.slot, b.load, b.dye)
+    e = lambda *s_, dt=torch.bfloat16: torch.empty(s_, dtype=dt, device="cuda")  # noqa: E731
+    qkv, o, ye, lse = e(G, C, 3 * hd), e(G, C, hd), e(G, C, d), e(G, H, C, dt=torch.float32)
+    dxe, dwqkv, dwo = e(G, C, d), e(G, d, 3 * hd), e(G, hd, d)
+    ws = torch.empty(vm.vmoe_attn_expert_bwd_workspace_size(p, H), dtype=torch.uint8, device="cuda")
+    vm.vmoe_attn_expert_fwd(p, H, b.xe, wqkv, wo, b.load, qkv, o, lse, ye)
+    vm.vmoe_attn_expert_bwd(p, H, b.xe, qkv, o, lse, wqkv, wo, b.dye, b.load, dxe, dwqkv, dwo, ws)
+    torch.cuda.synchronize()
+    assert vm.vmoe_device_status() == 0
+    load = b.load.cpu().numpy().reshape(-1)
+    assert C <= 128  # the fused backward, as in the benchmark
+    picks = sorted({0, G // 2, G - 1, int(np.argmax(load)), int(np.argmin(load))})
+    rows = valid_rows(load.reshape(T, E), C).reshape(G, C)[picks]
+    _compare_stages("attn_vitb_t17_sampled", H, load[picks], rows,
+                    _host(picks, G, C, d, H, b, qkv, o, ye, lse, ws, dxe, dwqkv, dwo, wqkv, wo))
